@@ -1,0 +1,23 @@
+import os
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+
+def pytest_configure(config):
+    config.addinivalue_line("markers", "gpu: needs a CUDA GPU (GB300, sm_103a)")
+    config.addinivalue_line("markers", "slow: long-running (large model sizes)")
+
+
+@pytest.fixture(scope="session")
+def built():
+    """Build the oracle and the host generator (CPU only)."""
+    from oracle import build as ob
+    from synth import build as sb
+    ob.build()
+    sb.build_host()
+    return True
