@@ -1,0 +1,415 @@
+"""Benchmark of the target-side block verification step on GB300.
+
+Default workload (one JSON line): the 7B-class decoder (28 layers, hidden
+3584, 28/4 heads, head_dim 128, FFN 18944, vocab 152064, bf16 random-init
+weights), one request whose cache holds 1564 prefilled positions (60 s of
+audio at 25 tokens/s plus 64 instruction tokens), candidate blocks of k = 8
+whose accepted length is geometric with mean 3 (capped at k), 256
+consecutive verification blocks.  A step is one verification block: the
+whole hot path (embedding, 28 layers, LM head + argmax, accept scan and
+rollback) through the C-ABI.
+
+value  = committed tokens / s over the timed blocks (inputs resident in HBM).
+e2e    = the same metric through the C-ABI with host buffers: each block's
+         candidates copied host->device and its (n_accepted, correction)
+         copied device->host inside the timed region.
+--impl reference times the CPU oracle on the same workload instead.
+"""
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "7B verify-step µs & committed tok/s vs block k; fraction of HBM roofline"
+UNIT = "committed tok/s"
+WORKLOAD = "7b"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=256)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--k", type=int, default=8)
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--profile-class", default="gate_up")
+    ap.add_argument("--model", default="7b", help="model shape (7b; smaller ones for quick checks)")
+    ap.add_argument("--kv-len", type=int, default=1564)
+    return ap.parse_args()
+
+
+def dist_setup(args):
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def load_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons while running."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.Q}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except Exception:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.strip().splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def model_shape(name):
+    from synth import workloads as W
+    return W.MODELS[name]
+
+
+def draw_plans(args, steps, vocab):
+    from synth import workloads as W
+    rng = np.random.default_rng(args.seed + 17)
+    return np.stack([W.geometric_plan(rng, args.k, vocab) for _ in range(steps)])
+
+
+def bytes_per_block(cfg, L, k):
+    """Algorithmic HBM bytes of one block: every weight once plus the KV read
+    by attention (all layers), as the roofline of the workload defines it."""
+    return cfg.weight_bytes() + (L + k + 1) * cfg.kv_bytes_per_pos()
+
+
+def run_ours(args, ws, rank, local):
+    import torch
+    import torch.distributed as dist
+
+    import paper_2609_37617_gb300 as lib
+    import synth
+    from synth import device as D
+    from synth import workloads as W
+
+    torch.cuda.set_device(local)
+    if ws > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    cfg = model_shape(args.model)
+    k, L0, steps, warm = args.k, args.kv_len, args.steps, args.warmup
+    seed = args.seed + rank
+    stream = torch.cuda.Stream()
+    sh = stream.cuda_stream
+
+    with torch.cuda.stream(stream):
+        dev_w = D.device_weights(cfg, seed)
+        torch.cuda.synchronize()
+        model = lib.Model(cfg, D.weight_pointers(cfg, dev_w))
+        del dev_w
+        torch.cuda.empty_cache()
+        plans = draw_plans(args, steps, cfg.vocab)
+        committed_plan = int((plans[:, 0] + 1).sum())
+        traj_len = committed_plan + k + 2
+        cap = L0 + (k + 1) * max(steps, warm) + traj_len + 64
+        kc, vc = D.device_kv(cfg, [L0], cap, seed, poison=False)
+        root0 = int(W.root_tokens(cfg, 1, seed)[0])
+        state = lib.State(model, [L0], cap, kc, vc, [root0])
+        len_dev, _ = state.device_state()
+
+        # greedy trajectory from the initial state (untimed), on the device
+        traj = torch.zeros(traj_len + 1, dtype=torch.int32, device="cuda")
+        traj[0] = root0
+        nbuf = torch.zeros(1, dtype=torch.int32, device="cuda")
+        for j in range(traj_len):
+            out = lib.make_verify_out(nbuf.data_ptr(), traj.data_ptr() + 4 * (j + 1))
+            lib._check(lib.as2d_decode_step(state.handle, out, sh), "as2d_decode_step")
+        state.check(sh)
+        state.rollback([L0], [root0], sh)
+        state.read_state(sh)
+
+        plans_d = torch.from_numpy(plans.astype(np.int32)).cuda()
+        cand = torch.zeros(k, dtype=torch.int32, device="cuda")
+        n_all = torch.zeros(steps, dtype=torch.int32, device="cuda")
+        c_all = torch.zeros(steps, dtype=torch.int32, device="cuda")
+
+        def block(i, plan_row):
+            rc = synth._load_cuda().synth_cuda_build_candidates(
+                cand.data_ptr(), traj.data_ptr(), traj_len + 1, len_dev, L0,
+                plans_d[plan_row].data_ptr(), k, cfg.vocab, sh)
+            assert rc == 0
+            out = lib.make_verify_out(n_all.data_ptr() + 4 * i, c_all.data_ptr() + 4 * i)
+            lib._check(lib.as2d_verify_block(state.handle, cand.data_ptr(), [k], out, sh),
+                       "as2d_verify_block")
+
+        for w in range(warm):
+            block(w % steps, w % steps)
+        state.check(sh)
+        state.rollback([L0], [root0], sh)
+        state.read_state(sh)
+        n_all.zero_()
+
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(steps)]
+        t0 = torch.cuda.Event(enable_timing=True)
+        t1 = torch.cuda.Event(enable_timing=True)
+        state.profile(args.profile_class)
+        state.profile_read()
+        clocks = ClockSampler(local)
+        clocks.start()
+        time.sleep(0.3)
+        if ws > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+        t0.record(stream)
+        for i in range(steps):
+            ev[i][0].record(stream)
+            block(i, i)
+            ev[i][1].record(stream)
+        t1.record(stream)
+        torch.cuda.synchronize()
+        if ws > 1:
+            dist.barrier()
+        clk = clocks.stop()
+        prof_n, prof_ms, all_launches = state.profile_read()
+        state.profile(None)
+        state.check(sh)
+        elapsed_ms = t0.elapsed_time(t1)
+        per_block_us = np.array([a.elapsed_time(b) * 1e3 for a, b in ev])
+        n_np = n_all.cpu().numpy()
+        committed = int((n_np + 1).sum())
+        plan_match = float(np.mean(n_np == plans[:, 0]))
+
+        e2e = None
+        if not args.no_e2e:
+            e2e = run_e2e(args, lib, W, state, traj, plans, cfg, L0, root0, sh, stream)
+
+    if ws > 1:
+        t = torch.tensor([elapsed_ms, committed], dtype=torch.float64, device="cuda")
+        mx = t.clone()
+        dist.all_reduce(mx, op=dist.ReduceOp.MAX)
+        sm = t.clone()
+        dist.all_reduce(sm, op=dist.ReduceOp.SUM)
+        elapsed_ms, committed_all = float(mx[0]), float(sm[1])
+    else:
+        committed_all = committed
+    value = committed_all / (elapsed_ms / 1e3)
+    peak, peak_kind = load_peaks()
+
+    # roofline of the dominant kernel class (per layer: one pair of events)
+    H, F = cfg.hidden, cfg.ffn
+    rows = k + 1
+    cls = args.profile_class
+    per_unit = {
+        "gate_up": 2 * F * H * 2 + rows * (H * 4 + 2 * H * 2 + F * 2),
+        "down": H * F * 2 + rows * (F * 2 + 2 * H * 4),
+        "qkv": (cfg.n_q + 2 * cfg.n_kv) * cfg.head_dim * H * 2 + rows * (H * 4 + 2 * H * 2),
+        "o": H * cfg.n_q * cfg.head_dim * 2 + rows * (cfg.n_q * cfg.head_dim * 2 + 2 * H * 4),
+        "lm_head": cfg.vocab * H * 2 + rows * (H * 4 + 2 * H * 2),
+    }.get(cls)
+    roofline = None
+    if prof_n and per_unit:
+        avg_ms = prof_ms / prof_n
+        achieved = per_unit / (avg_ms / 1e3) / 1e9
+        roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
+                    "unit": "GB/s", "frac": round(achieved / peak, 4),
+                    "traffic": None, "kernel": cls, "peak_kind": peak_kind,
+                    "launches": prof_n, "avg_us": round(avg_ms * 1e3, 2),
+                    "bytes_per_launch": int(per_unit)}
+    step_bytes = bytes_per_block(cfg, L0 + committed / 2.0, k)  # mean length over the blocks
+    med_us = float(np.median(per_block_us))
+    step_roof = {"bytes_per_block": int(step_bytes),
+                 "roofline_us": round(step_bytes / (peak * 1e9) * 1e6, 1),
+                 "frac_of_median_block": round(step_bytes / (peak * 1e9) / (med_us / 1e6), 4)}
+
+    line = {
+        "metric": METRIC, "value": round(value, 2), "unit": UNIT, "n_gpus": ws,
+        "steps": steps, "warmup": warm, "ms_per_step": round(elapsed_ms / steps, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16", "data": "synthetic (seeded random-init weights and KV; greedy-derived candidates)",
+        "config": {"workload": f"{args.model} verify, k={k}, L0={L0}, {steps} consecutive blocks, "
+                               "geometric acceptance (mean 3, capped at k)",
+                   "k": k, "kv_len": L0, "blocks": steps, "batch": 1,
+                   "l2": "inputs larger than L2 (14.1 GB of weights streamed per step)",
+                   "parallelism": f"replicas x{ws}" if ws > 1 else "single GPU"},
+        "verify_us": {"median": round(med_us, 1), "p10": round(float(np.percentile(per_block_us, 10)), 1),
+                      "p90": round(float(np.percentile(per_block_us, 90)), 1)},
+        "mean_committed_per_block": round(committed / steps, 3),
+        "plan_match": plan_match,
+        "step_roofline": step_roof,
+        "roofline": roofline,
+        "gpu_launches": int(all_launches),
+        "clocks": clk,
+        "e2e": e2e,
+    }
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(args, cfg, L0, plans)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    state.close()
+    model.close()
+    if ws > 1:
+        dist.destroy_process_group()
+
+
+def run_e2e(args, lib, W, state, traj, plans, cfg, L0, root0, sh, stream):
+    """Host-buffer loop through the C-ABI: per block, host candidates ->
+    device, verify, (n_accepted, correction) -> host, host bookkeeping."""
+    import torch
+    k = args.k
+    state.rollback([L0], [root0], sh)
+    state.read_state(sh)
+    traj_h = traj.cpu().numpy()
+    cand_h = torch.zeros(k, dtype=torch.int32).pin_memory()
+    out_h = torch.zeros(2, dtype=torch.int32).pin_memory()
+    cand_d = torch.zeros(k, dtype=torch.int32, device="cuda")
+    out_d = torch.zeros(2, dtype=torch.int32, device="cuda")
+    steps = min(args.steps, len(plans))
+    m = 0
+    committed = 0
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for i in range(steps):
+        cand_h.numpy()[:] = W.apply_plan(traj_h[m + 1:m + 1 + k], plans[i], cfg.vocab)
+        cand_d.copy_(cand_h, non_blocking=True)
+        out = lib.make_verify_out(out_d.data_ptr(), out_d.data_ptr() + 4)
+        lib._check(lib.as2d_verify_block(state.handle, cand_d.data_ptr(), [k], out, sh),
+                   "as2d_verify_block")
+        out_h.copy_(out_d, non_blocking=True)
+        stream.synchronize()
+        n = int(out_h[0])
+        m += n + 1
+        committed += n + 1
+    t1 = time.perf_counter()
+    state.check(sh)
+    return {"value": round(committed / (t1 - t0), 2), "unit": UNIT,
+            "h2d_bytes_per_step": 4 * k, "d2h_bytes_per_step": 8, "steps": steps}
+
+
+def cpu_baseline(args, cfg, L0, plans):
+    """The CPU oracle (as it stands) on one verification block of the same
+    workload: one k-block forward at L0 on the host cores."""
+    import oracle
+    from synth import workloads as W
+    k = args.k
+    hw = W.host_weights(cfg, args.seed)
+    om = oracle.Model(cfg, hw)
+    ks, vs = W.host_kv_request(cfg, 0, L0, L0 + k + 8, args.seed, poison=False)
+    cache = om.cache(ks, vs)
+    root = int(W.root_tokens(cfg, 1, args.seed)[0])
+    cand = plans[0, 2:2 + k]
+    t0 = time.perf_counter()
+    om.verify_block(cache, L0, root, cand, want_logits=False)
+    dt = time.perf_counter() - t0
+    mean_committed = float((plans[:, 0] + 1).mean())
+    cores = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    return {"value": round(mean_committed / dt, 4), "unit": UNIT, "cores": cores,
+            "kind": "oracle",
+            "sample": f"one k={k} verification block of the {cfg.name} decoder at L={L0} "
+                      f"({dt:.2f} s, fp64, OpenMP); value = mean committed tokens per block "
+                      "of the timed plan / that block time"}
+
+
+def run_reference(args, ws, rank):
+    """The CPU oracle timed as the reference arm: each step is one of the
+    k+1 rows of a verification block (one decode step of the oracle)."""
+    if rank != 0:
+        return
+    import oracle
+    from synth import workloads as W
+    cfg = model_shape(args.model)
+    k, L0 = args.k, args.kv_len
+    steps, warm = args.steps, args.warmup
+    hw = W.host_weights(cfg, args.seed)
+    om = oracle.Model(cfg, hw)
+    cap = L0 + steps + warm + 8
+    ks, vs = W.host_kv_request(cfg, 0, L0, cap, args.seed, poison=False)
+    cache = om.cache(ks, vs)
+    plans = draw_plans(args, max(steps, 1), cfg.vocab)
+    tok = int(W.root_tokens(cfg, 1, args.seed)[0])
+    pos = L0
+    for _ in range(warm):
+        om.decode_step(cache, pos, tok)
+        pos += 1
+    t0 = time.perf_counter()
+    for i in range(steps):
+        om.decode_step(cache, pos, tok)
+        pos += 1
+    dt = time.perf_counter() - t0
+    rows_per_s = steps / dt
+    mean_committed = float((plans[:, 0] + 1).mean())
+    value = rows_per_s * mean_committed / (k + 1)
+    cores = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    line = {"impl": "reference", "metric": METRIC, "value": round(value, 4), "unit": UNIT,
+            "n_gpus": ws, "steps": steps, "warmup": warm,
+            "ms_per_step": round(dt / steps * 1e3, 3), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": f"{args.model} verify, k={k}, L0={L0}", "k": k, "kv_len": L0},
+            "cpu_baseline": {"value": round(value, 4), "unit": UNIT, "cores": cores,
+                             "kind": "oracle",
+                             "sample": f"each step = one of the {k + 1} rows of a k={k} block "
+                                       "(one oracle decode step); value = rows/s x mean "
+                                       "committed tokens per block / (k+1)"},
+            "e2e": {"value": round(value, 4), "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse()
+    ws, rank, local = dist_setup(args)
+    if args.impl == "reference":
+        run_reference(args, ws, rank)
+        return
+    run_ours(args, ws, rank, local)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,204 @@
+/*
+ * as2d.h -- C-ABI of the GB300 (sm_103a) target-side block verification
+ * library, libas2d.so.
+ *
+ * The operation (paper: Section 3.2 "Target verification"; App. A.2
+ * "Configuration and execution boundaries"; App. C.2 "Verification and state
+ * repair"; App. C.4, Eq. 3 and Prop. 1):
+ *   the target decoder holds a committed prefix in its KV cache (prefilled
+ *   audio and instruction tokens plus every committed token except the last
+ *   one) and a pending "known root" token -- the last committed token, not yet
+ *   forwarded.  A verification call forwards the root followed by k drafter
+ *   candidates c_1..c_k in one causal pass (physical width K = k + 1),
+ *   takes the greedy token g_i after each row i, accepts the longest prefix
+ *   c_1..c_n with c_{i+1} = g_i, and emits the correction g_n (the bonus
+ *   token when n = k).  The cache keeps the root's and the accepted
+ *   candidates' entries; the rejected rows' entries are dropped.  The
+ *   correction is not forwarded: it becomes the next call's root, so full
+ *   acceptance needs no extra single-token call (App. C.2, known-root
+ *   carry).  With k = 0 the call is one plain greedy decode
+ *   step of Eq. 3.
+ *
+ * Conventions shared by every entry point:
+ *   - Pointers documented "device" are CUDA device pointers on the current
+ *     device; "host" pointers are ordinary host memory, read before the call
+ *     returns.  `stream` is a cudaStream_t (NULL = the legacy default stream).
+ *   - Work is enqueued on `stream` and never synchronises with the host,
+ *     except where an entry point says it does.  Device outputs are valid once
+ *     the caller synchronises the stream.
+ *   - Argument errors are found on the host before anything is enqueued and
+ *     leave all state unchanged.  as2d_last_error() then describes the error
+ *     (thread-local).
+ *   - Every bf16 value is the upper 16 bits of an IEEE float (bfloat16).
+ */
+#ifndef AS2D_H
+#define AS2D_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef int32_t as2d_status;
+#define AS2D_OK 0
+#define AS2D_ERR_INVALID_ARG (-1)   /* bad pointer, size or value            */
+#define AS2D_ERR_CAPACITY (-2)      /* L + k + 1 would exceed the capacity   */
+#define AS2D_ERR_CUDA (-3)          /* a CUDA runtime call failed            */
+#define AS2D_ERR_UNSUPPORTED (-4)   /* shape outside what the kernels handle */
+#define AS2D_ERR_DEVICE (-5)        /* a kernel reported an error or timeout */
+
+/* Largest number of candidates per request in one call (the budget b of
+   App. A.2; physical width K = k + 1 <= 17). */
+#define AS2D_MAX_K 16
+/* Largest number of requests verified together in one call. */
+#define AS2D_MAX_BATCH 64
+
+/* Decoder shape.  Requirements: hidden % 128 == 0, (n_q * head_dim) % 128
+   == 0, ffn % 64 == 0, vocab % 8 == 0, head_dim in {64, 128},
+   n_q % n_kv == 0, n_kv * head_dim % 128 == 0.  rope_theta is the rotary base (rotate-half
+   pairing of dimensions i and i + head_dim/2, angle pos * theta^(-2i/d));
+   rms_eps is added to the mean square before the root. */
+typedef struct as2d_config {
+  int32_t n_layers, hidden, n_q_heads, n_kv_heads, head_dim, ffn, vocab;
+  float rope_theta, rms_eps;
+} as2d_config;
+
+/* Weights, as device pointers to bf16 in checkpoint (logical) layouts,
+   row-major: embed, lm_head [vocab][hidden]; final_norm and the per-layer
+   attn_norm, mlp_norm gains [hidden]; w_q [n_q*d][hidden], w_k, w_v
+   [n_kv*d][hidden] (head j in rows [j*d, (j+1)*d)); w_o [hidden][n_q*d];
+   w_gate, w_up [ffn][hidden]; w_down [hidden][ffn].  The per-layer members
+   are HOST arrays of n_layers device pointers.  as2d_model_load copies every
+   tensor into memory the model owns (re-laid out for the kernels); the caller
+   may free its buffers once as2d_model_load has returned. */
+typedef struct as2d_weights {
+  const void* embed;
+  const void* final_norm;
+  const void* lm_head;
+  const void* const* attn_norm;
+  const void* const* w_q;
+  const void* const* w_k;
+  const void* const* w_v;
+  const void* const* w_o;
+  const void* const* mlp_norm;
+  const void* const* w_gate;
+  const void* const* w_up;
+  const void* const* w_down;
+} as2d_weights;
+
+typedef struct as2d_model as2d_model;
+typedef struct as2d_kv as2d_kv;
+
+/* Outputs of one verification call.  rows = sum over requests of (k_b + 1),
+   ordered request by request, each request's root row first.
+   n_accepted, correction_token: device int32 [batch] (required).
+   greedy: device int32 [rows], the greedy token after each row (nullable).
+   logits: device float [rows][vocab], fp32 logits of every row (nullable;
+   the paper's full-logits verification of App. B.2 stores [1, K, vocab]). */
+typedef struct as2d_verify_out {
+  int32_t* n_accepted;
+  int32_t* correction_token;
+  int32_t* greedy;
+  float* logits;
+} as2d_verify_out;
+
+/* Load a model onto the current device.  Synchronises the device before it
+   returns.  On success *out owns its device memory until as2d_model_free. */
+as2d_status as2d_model_load(const as2d_config* cfg, const as2d_weights* w,
+                            as2d_model** out);
+
+/* Bind a verification state of `batch` requests to a caller-allocated cache
+   and its prefilled prefix (App. A.1: the retained audio KV plus the
+   instruction, a valid prefix of the reference prompt).
+   k_cache, v_cache: device bf16, layout [n_layers][batch][n_kv][capacity]
+   [head_dim]; positions [0, kv_len[b]) of request b hold its prefilled keys
+   (already rotated to their positions) and values.  The library writes the
+   entries of forwarded rows; the caller keeps both buffers alive until
+   as2d_kv_free.  kv_len, root_tokens: host int32 [batch]; root_tokens[b] is
+   request b's pending known root (the first token chosen after prefill).
+   Allocates the state's device working memory.  Synchronises the device. */
+as2d_status as2d_kv_init_prefilled(as2d_model* model, int32_t batch,
+                                   const int32_t* kv_len, int32_t capacity,
+                                   void* k_cache, void* v_cache,
+                                   const int32_t* root_tokens, as2d_kv** out);
+
+/* Verify one block per request (Section 3.2; App. C.2).
+   candidates: device int32, packed: request b's k_b candidates start at
+   index sum_{b' < b} k_{b'}.  k: host int32 [batch], 0 <= k_b <= AS2D_MAX_K.
+   Request b forwards rows [root_b, c_1..c_{k_b}] at positions
+   L_b .. L_b + k_b and afterwards holds L_b' = L_b + n_b + 1 and
+   root_b' = correction_b, all on the device.  The host keeps only an upper
+   bound of L_b (it grows by k_b + 1 per call); AS2D_ERR_CAPACITY is returned
+   when that bound plus k_b + 1 would exceed the capacity (as2d_kv_read_state
+   refreshes the bound).  Candidate ids outside [0, vocab) are a device-side
+   error (as2d_kv_check).  Results are batch invariant: each row's logits are
+   bitwise the same whatever the other rows of the call. */
+as2d_status as2d_verify_block(as2d_kv* kv, const int32_t* candidates,
+                              const int32_t* k, const as2d_verify_out* out,
+                              void* stream);
+
+/* One greedy decode step for every request: as2d_verify_block with all
+   k_b = 0 (App. C.2: with no ready candidate the target advances alone by one
+   token). */
+as2d_status as2d_decode_step(as2d_kv* kv, const as2d_verify_out* out,
+                             void* stream);
+
+/* Restore each request's state to an earlier committed prefix (App. C.4,
+   requirement 2): length new_len[b] and pending root new_root[b] (host int32
+   [batch]).  Entries [0, new_len[b]) must be ones this state holds; a
+   new_len above the device-side length is a device error that leaves that
+   request unchanged.  Asynchronous on `stream`. */
+as2d_status as2d_kv_rollback(as2d_kv* kv, const int32_t* new_len,
+                             const int32_t* new_root, void* stream);
+
+/* Synchronise `stream`, copy the device-side lengths and roots into host
+   int32 [batch] arrays (either may be NULL) and reset the host's length
+   bounds to them. */
+as2d_status as2d_kv_read_state(as2d_kv* kv, int32_t* len, int32_t* root,
+                               void* stream);
+
+/* Device pointers to the state's int32 [batch] lengths and roots, for
+   consumers on the device (e.g. a drafter kernel that builds the next block
+   without a host round trip).  Read-only for the caller. */
+as2d_status as2d_kv_device_state(as2d_kv* kv, const int32_t** len,
+                                 const int32_t** root);
+
+/* Synchronise `stream` and return AS2D_ERR_DEVICE if any kernel of this
+   state reported an error since the last check (then cleared), else
+   AS2D_OK. */
+as2d_status as2d_kv_check(as2d_kv* kv, void* stream);
+
+/* Measurement support (not part of the verification step).  Kernel classes
+   of one verification pass, in launch order per layer: */
+#define AS2D_KERNEL_QKV 0        /* norm + QKV projection               */
+#define AS2D_KERNEL_ATTENTION 1  /* RoPE + KV append + attention        */
+#define AS2D_KERNEL_O 2          /* output projection + residual        */
+#define AS2D_KERNEL_GATE_UP 3    /* norm + gate/up projection + SwiGLU   */
+#define AS2D_KERNEL_DOWN 4       /* down projection + residual          */
+#define AS2D_KERNEL_LM_HEAD 5    /* final norm + LM head + argmax       */
+#define AS2D_KERNEL_OTHER 6      /* embedding gather, accept scan, ...  */
+#define AS2D_KERNEL_CLASSES 7
+
+/* Record a CUDA event pair on the call's stream around the launches of
+   kernel class `kernel_class` (one pair per layer, or per call for the LM
+   head) in later calls (-1 stops recording).  Also
+   counts every kernel the library launches.  Events are created on demand. */
+as2d_status as2d_kv_profile(as2d_kv* kv, int32_t kernel_class);
+
+/* Synchronise the recorded events and return the number of recorded
+   event pairs of the class, their summed device time in milliseconds, and the
+   number of kernels of any class launched since the last read; then reset. */
+as2d_status as2d_kv_profile_read(as2d_kv* kv, int32_t* launches,
+                                 double* total_ms, int64_t* all_launches);
+
+void as2d_kv_free(as2d_kv* kv);
+void as2d_model_free(as2d_model* model);
+
+/* Thread-local description of the last error ("" if none). */
+const char* as2d_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif

@@ -1,0 +1,296 @@
+"""Python binding of libas2d.so, the GB300 (sm_103a) target-side block
+verification library (C-ABI: include/as2d.h).
+
+The functions below carry the C names and only marshal arguments: every step
+of the verification pass runs in the library's CUDA kernels.  PyTorch is used
+by callers for device memory and streams only.  Importing this package fails
+loudly if libas2d.so has not been built: there is no fallback path.
+"""
+import ctypes
+import os
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libas2d.so")
+
+if not os.path.exists(LIB_PATH):
+    raise ImportError(
+        f"{LIB_PATH} is missing: build it with __graft_entry__.build() "
+        "(or python paper_2609_37617_gb300/build.py). There is no CPU fallback.")
+
+_lib = ctypes.CDLL(LIB_PATH)
+
+AS2D_OK = 0
+AS2D_ERR_INVALID_ARG = -1
+AS2D_ERR_CAPACITY = -2
+AS2D_ERR_CUDA = -3
+AS2D_ERR_UNSUPPORTED = -4
+AS2D_ERR_DEVICE = -5
+AS2D_MAX_K = 16
+AS2D_MAX_BATCH = 64
+
+EXPORTED = ("as2d_model_load", "as2d_kv_init_prefilled", "as2d_verify_block",
+            "as2d_decode_step", "as2d_kv_rollback", "as2d_kv_read_state",
+            "as2d_kv_device_state", "as2d_kv_check", "as2d_kv_free",
+            "as2d_model_free", "as2d_last_error", "as2d_kv_profile",
+            "as2d_kv_profile_read")
+KERNEL_CLASSES = {"qkv": 0, "attention": 1, "o": 2, "gate_up": 3, "down": 4,
+                  "lm_head": 5, "other": 6}
+
+
+class as2d_config(ctypes.Structure):
+    _fields_ = [("n_layers", ctypes.c_int32), ("hidden", ctypes.c_int32),
+                ("n_q_heads", ctypes.c_int32), ("n_kv_heads", ctypes.c_int32),
+                ("head_dim", ctypes.c_int32), ("ffn", ctypes.c_int32),
+                ("vocab", ctypes.c_int32), ("rope_theta", ctypes.c_float),
+                ("rms_eps", ctypes.c_float)]
+
+
+class as2d_weights(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in (
+        "embed", "final_norm", "lm_head", "attn_norm", "w_q", "w_k", "w_v",
+        "w_o", "mlp_norm", "w_gate", "w_up", "w_down")]
+
+
+class as2d_verify_out(ctypes.Structure):
+    _fields_ = [("n_accepted", ctypes.c_void_p), ("correction_token", ctypes.c_void_p),
+                ("greedy", ctypes.c_void_p), ("logits", ctypes.c_void_p)]
+
+
+_P = ctypes.c_void_p
+_S = ctypes.c_int32
+_lib.as2d_model_load.argtypes = [ctypes.POINTER(as2d_config), ctypes.POINTER(as2d_weights),
+                                 ctypes.POINTER(ctypes.c_void_p)]
+_lib.as2d_model_load.restype = _S
+_lib.as2d_kv_init_prefilled.argtypes = [_P, ctypes.c_int32, _P, ctypes.c_int32, _P, _P, _P,
+                                        ctypes.POINTER(ctypes.c_void_p)]
+_lib.as2d_kv_init_prefilled.restype = _S
+_lib.as2d_verify_block.argtypes = [_P, _P, _P, ctypes.POINTER(as2d_verify_out), _P]
+_lib.as2d_verify_block.restype = _S
+_lib.as2d_decode_step.argtypes = [_P, ctypes.POINTER(as2d_verify_out), _P]
+_lib.as2d_decode_step.restype = _S
+_lib.as2d_kv_rollback.argtypes = [_P, _P, _P, _P]
+_lib.as2d_kv_rollback.restype = _S
+_lib.as2d_kv_read_state.argtypes = [_P, _P, _P, _P]
+_lib.as2d_kv_read_state.restype = _S
+_lib.as2d_kv_device_state.argtypes = [_P, ctypes.POINTER(ctypes.c_void_p),
+                                      ctypes.POINTER(ctypes.c_void_p)]
+_lib.as2d_kv_device_state.restype = _S
+_lib.as2d_kv_check.argtypes = [_P, _P]
+_lib.as2d_kv_check.restype = _S
+_lib.as2d_kv_free.argtypes = [_P]
+_lib.as2d_kv_free.restype = None
+_lib.as2d_model_free.argtypes = [_P]
+_lib.as2d_model_free.restype = None
+_lib.as2d_kv_profile.argtypes = [_P, ctypes.c_int32]
+_lib.as2d_kv_profile.restype = _S
+_lib.as2d_kv_profile_read.argtypes = [_P, ctypes.POINTER(ctypes.c_int32),
+                                      ctypes.POINTER(ctypes.c_double),
+                                      ctypes.POINTER(ctypes.c_int64)]
+_lib.as2d_kv_profile_read.restype = _S
+_lib.as2d_last_error.argtypes = []
+_lib.as2d_last_error.restype = ctypes.c_char_p
+
+
+class AS2DError(RuntimeError):
+    def __init__(self, status, where):
+        msg = _lib.as2d_last_error().decode(errors="replace")
+        super().__init__(f"{where} returned {status}: {msg}")
+        self.status = status
+
+
+def _check(status, where):
+    if status != AS2D_OK:
+        raise AS2DError(status, where)
+    return status
+
+
+def _i32_array(values):
+    arr = (ctypes.c_int32 * len(values))(*[int(v) for v in values])
+    return arr
+
+
+# ---- the C entry points, one wrapper each -------------------------------------
+
+def as2d_last_error():
+    return _lib.as2d_last_error().decode(errors="replace")
+
+
+def as2d_model_load(cfg, weights_ptrs, n_layers):
+    """cfg: as2d_config; weights_ptrs: dict name -> device pointer (int) for
+    embed/final_norm/lm_head and name -> list of n_layers pointers for the
+    per-layer tensors.  Returns (status, model handle)."""
+    keep = []
+    w = as2d_weights()
+    for name in ("embed", "final_norm", "lm_head"):
+        setattr(w, name, int(weights_ptrs[name]))
+    for name in ("attn_norm", "w_q", "w_k", "w_v", "w_o", "mlp_norm", "w_gate",
+                 "w_up", "w_down"):
+        arr = (ctypes.c_void_p * n_layers)(*[int(p) for p in weights_ptrs[name]])
+        keep.append(arr)
+        setattr(w, name, ctypes.cast(arr, ctypes.c_void_p).value)
+    out = ctypes.c_void_p()
+    st = _lib.as2d_model_load(ctypes.byref(cfg), ctypes.byref(w), ctypes.byref(out))
+    return st, out.value
+
+
+def as2d_kv_init_prefilled(model, batch, kv_len, capacity, k_cache_ptr, v_cache_ptr,
+                           root_tokens):
+    out = ctypes.c_void_p()
+    st = _lib.as2d_kv_init_prefilled(_P(model), int(batch), _i32_array(kv_len),
+                                     int(capacity), _P(int(k_cache_ptr)),
+                                     _P(int(v_cache_ptr)), _i32_array(root_tokens),
+                                     ctypes.byref(out))
+    return st, out.value
+
+
+def make_verify_out(n_accepted_ptr, correction_ptr, greedy_ptr=0, logits_ptr=0):
+    return as2d_verify_out(int(n_accepted_ptr) or None, int(correction_ptr) or None,
+                           int(greedy_ptr) or None, int(logits_ptr) or None)
+
+
+def as2d_verify_block(kv, candidates_ptr, k, out, stream=0):
+    return _lib.as2d_verify_block(_P(kv), _P(int(candidates_ptr) or None), _i32_array(k),
+                                  ctypes.byref(out), _P(int(stream) or None))
+
+
+def as2d_decode_step(kv, out, stream=0):
+    return _lib.as2d_decode_step(_P(kv), ctypes.byref(out), _P(int(stream) or None))
+
+
+def as2d_kv_rollback(kv, new_len, new_root, stream=0):
+    return _lib.as2d_kv_rollback(_P(kv), _i32_array(new_len), _i32_array(new_root),
+                                 _P(int(stream) or None))
+
+
+def as2d_kv_read_state(kv, batch, stream=0):
+    ln = (ctypes.c_int32 * batch)()
+    rt = (ctypes.c_int32 * batch)()
+    st = _lib.as2d_kv_read_state(_P(kv), ln, rt, _P(int(stream) or None))
+    return st, list(ln), list(rt)
+
+
+def as2d_kv_device_state(kv):
+    ln = ctypes.c_void_p()
+    rt = ctypes.c_void_p()
+    st = _lib.as2d_kv_device_state(_P(kv), ctypes.byref(ln), ctypes.byref(rt))
+    return st, ln.value, rt.value
+
+
+def as2d_kv_check(kv, stream=0):
+    return _lib.as2d_kv_check(_P(kv), _P(int(stream) or None))
+
+
+def as2d_kv_free(kv):
+    _lib.as2d_kv_free(_P(kv))
+
+
+def as2d_model_free(model):
+    _lib.as2d_model_free(_P(model))
+
+
+def as2d_kv_profile(kv, kernel_class):
+    return _lib.as2d_kv_profile(_P(kv), int(kernel_class))
+
+
+def as2d_kv_profile_read(kv):
+    n = ctypes.c_int32()
+    ms = ctypes.c_double()
+    alln = ctypes.c_int64()
+    st = _lib.as2d_kv_profile_read(_P(kv), ctypes.byref(n), ctypes.byref(ms), ctypes.byref(alln))
+    return st, n.value, ms.value, alln.value
+
+
+def exported_symbols():
+    """Names of include/as2d.h's entry points that the loaded library exports."""
+    return [n for n in EXPORTED if hasattr(_lib, n)]
+
+
+# ---- thin owners of the handles (marshalling only) ---------------------------
+
+class Model:
+    """Owns an as2d_model.  `shape` has the fields of as2d_config
+    (n_layers, hidden, n_q, n_kv, head_dim, ffn, vocab, rope_theta, rms_eps);
+    `pointers` maps weight names to device pointers (see as2d_model_load)."""
+
+    def __init__(self, shape, pointers):
+        self.shape = shape
+        self.cfg = as2d_config(shape.n_layers, shape.hidden, shape.n_q, shape.n_kv,
+                               shape.head_dim, shape.ffn, shape.vocab,
+                               float(shape.rope_theta), float(shape.rms_eps))
+        st, h = as2d_model_load(self.cfg, pointers, shape.n_layers)
+        _check(st, "as2d_model_load")
+        self.handle = h
+
+    def close(self):
+        if self.handle:
+            as2d_model_free(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+class State:
+    """Owns an as2d_kv bound to caller caches (torch tensors kept alive here)."""
+
+    def __init__(self, model, kv_len, capacity, k_cache, v_cache, roots):
+        self.model = model
+        self.batch = len(kv_len)
+        self._caches = (k_cache, v_cache)
+        st, h = as2d_kv_init_prefilled(model.handle, self.batch, kv_len, capacity,
+                                       k_cache.data_ptr(), v_cache.data_ptr(), roots)
+        _check(st, "as2d_kv_init_prefilled")
+        self.handle = h
+
+    def verify(self, candidates, k, n_accepted, correction, greedy=None, logits=None,
+               stream=0):
+        out = make_verify_out(n_accepted.data_ptr(), correction.data_ptr(),
+                              greedy.data_ptr() if greedy is not None else 0,
+                              logits.data_ptr() if logits is not None else 0)
+        cptr = candidates.data_ptr() if candidates is not None and candidates.numel() else 0
+        _check(as2d_verify_block(self.handle, cptr, k, out, stream), "as2d_verify_block")
+
+    def decode(self, n_accepted, correction, greedy=None, logits=None, stream=0):
+        out = make_verify_out(n_accepted.data_ptr(), correction.data_ptr(),
+                              greedy.data_ptr() if greedy is not None else 0,
+                              logits.data_ptr() if logits is not None else 0)
+        _check(as2d_decode_step(self.handle, out, stream), "as2d_decode_step")
+
+    def rollback(self, new_len, new_root, stream=0):
+        _check(as2d_kv_rollback(self.handle, new_len, new_root, stream), "as2d_kv_rollback")
+
+    def read_state(self, stream=0):
+        st, ln, rt = as2d_kv_read_state(self.handle, self.batch, stream)
+        _check(st, "as2d_kv_read_state")
+        return ln, rt
+
+    def device_state(self):
+        st, ln, rt = as2d_kv_device_state(self.handle)
+        _check(st, "as2d_kv_device_state")
+        return ln, rt
+
+    def profile(self, kernel_class):
+        cls = KERNEL_CLASSES[kernel_class] if isinstance(kernel_class, str) else kernel_class
+        _check(as2d_kv_profile(self.handle, -1 if cls is None else cls), "as2d_kv_profile")
+
+    def profile_read(self):
+        st, n, ms, alln = as2d_kv_profile_read(self.handle)
+        _check(st, "as2d_kv_profile_read")
+        return n, ms, alln
+
+    def check(self, stream=0):
+        _check(as2d_kv_check(self.handle, stream), "as2d_kv_check")
+
+    def close(self):
+        if self.handle:
+            as2d_kv_free(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

@@ -1,0 +1,442 @@
+// as2d_api.cu -- the C-ABI of include/as2d.h: argument checking, ownership,
+// weight re-layout at load time, and the per-call launch sequence of the
+// verification pass (Section 3.2; App. C.2).
+#include <cstring>
+#include <string>
+
+#include "as2d_internal.h"
+
+using namespace as2d;
+
+struct as2d_model {
+  Model m;
+};
+struct as2d_kv {
+  KvState s;
+};
+
+namespace {
+
+thread_local std::string g_err;
+
+as2d_status fail(as2d_status st, const std::string& msg) {
+  g_err = msg;
+  return st;
+}
+
+#define CUDA_TRY(expr)                                                      \
+  do {                                                                      \
+    cudaError_t e_ = (expr);                                                \
+    if (e_ != cudaSuccess)                                                  \
+      return fail(AS2D_ERR_CUDA, std::string(#expr) + ": " +                \
+                                     cudaGetErrorString(e_));               \
+  } while (0)
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// Carves consecutive 256-byte-aligned pieces out of one allocation.
+struct Carver {
+  char* base;
+  size_t off = 0;
+  template <typename T>
+  T* take(size_t count) {
+    off = align_up(off, 256);
+    T* p = reinterpret_cast<T*>(base + off);
+    off += count * sizeof(T);
+    return p;
+  }
+};
+
+as2d_status check_config(const as2d_config* c) {
+  if (!c) return fail(AS2D_ERR_INVALID_ARG, "config is NULL");
+  if (c->n_layers <= 0 || c->hidden <= 0 || c->n_q_heads <= 0 ||
+      c->n_kv_heads <= 0 || c->head_dim <= 0 || c->ffn <= 0 || c->vocab <= 1)
+    return fail(AS2D_ERR_INVALID_ARG, "config sizes must be positive");
+  if (!(c->rope_theta > 0.f) || !(c->rms_eps >= 0.f))
+    return fail(AS2D_ERR_INVALID_ARG, "rope_theta must be > 0 and rms_eps >= 0");
+  if (c->n_q_heads % c->n_kv_heads != 0)
+    return fail(AS2D_ERR_INVALID_ARG, "n_q_heads must be a multiple of n_kv_heads");
+  if (c->head_dim != 64 && c->head_dim != 128)
+    return fail(AS2D_ERR_UNSUPPORTED, "head_dim must be 64 or 128");
+  if (c->hidden % 128 != 0 || (c->n_q_heads * c->head_dim) % 128 != 0 ||
+      (c->n_kv_heads * c->head_dim) % 128 != 0)
+    return fail(AS2D_ERR_UNSUPPORTED,
+                "hidden, n_q*head_dim and n_kv*head_dim must be multiples of 128");
+  if (c->ffn % 64 != 0) return fail(AS2D_ERR_UNSUPPORTED, "ffn must be a multiple of 64");
+  if (c->vocab % 8 != 0) return fail(AS2D_ERR_UNSUPPORTED, "vocab must be a multiple of 8");
+  return AS2D_OK;
+}
+
+}  // namespace
+
+extern "C" const char* as2d_last_error(void) { return g_err.c_str(); }
+
+extern "C" as2d_status as2d_model_load(const as2d_config* cfg,
+                                       const as2d_weights* w,
+                                       as2d_model** out) {
+  g_err.clear();
+  as2d_status st = check_config(cfg);
+  if (st != AS2D_OK) return st;
+  if (!w || !out) return fail(AS2D_ERR_INVALID_ARG, "weights or out is NULL");
+  if (!w->embed || !w->final_norm || !w->lm_head || !w->attn_norm || !w->w_q ||
+      !w->w_k || !w->w_v || !w->w_o || !w->mlp_norm || !w->w_gate ||
+      !w->w_up || !w->w_down)
+    return fail(AS2D_ERR_INVALID_ARG, "a weight pointer is NULL");
+  const int L = cfg->n_layers;
+  for (int l = 0; l < L; ++l)
+    if (!w->attn_norm[l] || !w->w_q[l] || !w->w_k[l] || !w->w_v[l] ||
+        !w->w_o[l] || !w->mlp_norm[l] || !w->w_gate[l] || !w->w_up[l] ||
+        !w->w_down[l])
+      return fail(AS2D_ERR_INVALID_ARG, "a per-layer weight pointer is NULL");
+
+  as2d_model* mh = new as2d_model();
+  Model& m = mh->m;
+  m.cfg = *cfg;
+  const size_t H = cfg->hidden, F = cfg->ffn, V = cfg->vocab, d = cfg->head_dim;
+  m.q_dim = cfg->n_q_heads * cfg->head_dim;
+  m.kv_dim = cfg->n_kv_heads * cfg->head_dim;
+  m.qkv_rows = m.q_dim + 2 * m.kv_dim;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&m.sm_count, cudaDevAttrMultiProcessorCount, dev);
+  (void)d;
+
+  const size_t per_layer_bf16 = (size_t)m.qkv_rows * H + H * m.q_dim + 2 * F * H + H * F;
+  size_t bytes = 0;
+  bytes += align_up(V * H * 2, 256) * 2;
+  bytes += L * (align_up((size_t)m.qkv_rows * H * 2, 256) + align_up(H * m.q_dim * 2, 256) +
+                align_up(2 * F * H * 2, 256) + align_up(H * F * 2, 256) +
+                2 * align_up(H * 4, 256));
+  bytes += align_up(H * 4, 256) + 4096;
+  (void)per_layer_bf16;
+  cudaError_t e = cudaMalloc(&m.arena, bytes);
+  if (e != cudaSuccess) {
+    delete mh;
+    return fail(AS2D_ERR_CUDA, std::string("cudaMalloc of the weight arena: ") + cudaGetErrorString(e));
+  }
+  m.arena_bytes = bytes;
+  Carver cv{(char*)m.arena};
+  auto fail_free = [&](const std::string& msg) {
+    cudaFree(m.arena);
+    delete mh;
+    return fail(AS2D_ERR_CUDA, msg);
+  };
+#define LOAD_TRY(expr)                                                        \
+  do {                                                                        \
+    cudaError_t e_ = (expr);                                                  \
+    if (e_ != cudaSuccess)                                                    \
+      return fail_free(std::string(#expr) + ": " + cudaGetErrorString(e_));   \
+  } while (0)
+
+  bf16* embed = cv.take<bf16>(V * H);
+  bf16* lm = cv.take<bf16>(V * H);
+  float* fnorm = cv.take<float>(H);
+  LOAD_TRY(cudaMemcpy(embed, w->embed, V * H * 2, cudaMemcpyDeviceToDevice));
+  LOAD_TRY(cudaMemcpy(lm, w->lm_head, V * H * 2, cudaMemcpyDeviceToDevice));
+  LOAD_TRY(launch_f32_from_bf16(fnorm, w->final_norm, H, 0));
+  m.embed = embed;
+  m.lm_head = lm;
+  m.final_norm = fnorm;
+  for (int l = 0; l < L; ++l) {
+    bf16* qkv = cv.take<bf16>((size_t)m.qkv_rows * H);
+    bf16* wo = cv.take<bf16>(H * m.q_dim);
+    bf16* gu = cv.take<bf16>(2 * F * H);
+    bf16* wd = cv.take<bf16>(H * F);
+    float* an = cv.take<float>(H);
+    float* mn = cv.take<float>(H);
+    LOAD_TRY(cudaMemcpy(qkv, w->w_q[l], (size_t)m.q_dim * H * 2, cudaMemcpyDeviceToDevice));
+    LOAD_TRY(cudaMemcpy(qkv + (size_t)m.q_dim * H, w->w_k[l], (size_t)m.kv_dim * H * 2,
+                        cudaMemcpyDeviceToDevice));
+    LOAD_TRY(cudaMemcpy(qkv + (size_t)(m.q_dim + m.kv_dim) * H, w->w_v[l],
+                        (size_t)m.kv_dim * H * 2, cudaMemcpyDeviceToDevice));
+    LOAD_TRY(cudaMemcpy(wo, w->w_o[l], H * m.q_dim * 2, cudaMemcpyDeviceToDevice));
+    // gate/up interleaved in blocks of 64 rows: [64 gate | 64 up] per 128 rows
+    LOAD_TRY(cudaMemcpy2D(gu, 128 * H * 2, w->w_gate[l], 64 * H * 2, 64 * H * 2, F / 64,
+                          cudaMemcpyDeviceToDevice));
+    LOAD_TRY(cudaMemcpy2D(gu + 64 * H, 128 * H * 2, w->w_up[l], 64 * H * 2, 64 * H * 2, F / 64,
+                          cudaMemcpyDeviceToDevice));
+    LOAD_TRY(cudaMemcpy(wd, w->w_down[l], H * F * 2, cudaMemcpyDeviceToDevice));
+    LOAD_TRY(launch_f32_from_bf16(an, w->attn_norm[l], H, 0));
+    LOAD_TRY(launch_f32_from_bf16(mn, w->mlp_norm[l], H, 0));
+    m.w_qkv.push_back(qkv);
+    m.w_o.push_back(wo);
+    m.w_gu.push_back(gu);
+    m.w_down.push_back(wd);
+    m.attn_norm.push_back(an);
+    m.mlp_norm.push_back(mn);
+  }
+  LOAD_TRY(cudaDeviceSynchronize());
+#undef LOAD_TRY
+  *out = mh;
+  return AS2D_OK;
+}
+
+extern "C" void as2d_model_free(as2d_model* mh) {
+  if (!mh) return;
+  cudaFree(mh->m.arena);
+  delete mh;
+}
+
+extern "C" as2d_status as2d_kv_init_prefilled(as2d_model* mh, int32_t batch,
+                                              const int32_t* kv_len,
+                                              int32_t capacity, void* k_cache,
+                                              void* v_cache,
+                                              const int32_t* root_tokens,
+                                              as2d_kv** out) {
+  g_err.clear();
+  if (!mh || !kv_len || !k_cache || !v_cache || !root_tokens || !out)
+    return fail(AS2D_ERR_INVALID_ARG, "a pointer argument is NULL");
+  if (batch < 1 || batch > kMaxBatch)
+    return fail(AS2D_ERR_INVALID_ARG, "batch must be in [1, AS2D_MAX_BATCH]");
+  if (capacity < 1) return fail(AS2D_ERR_INVALID_ARG, "capacity must be positive");
+  const Model& m = mh->m;
+  for (int b = 0; b < batch; ++b) {
+    if (kv_len[b] < 0 || kv_len[b] >= capacity)
+      return fail(AS2D_ERR_CAPACITY, "kv_len must be in [0, capacity)");
+    if (root_tokens[b] < 0 || root_tokens[b] >= m.cfg.vocab)
+      return fail(AS2D_ERR_INVALID_ARG, "root token outside [0, vocab)");
+  }
+  as2d_kv* kh = new as2d_kv();
+  KvState& s = kh->s;
+  s.model = &mh->m;
+  s.batch = batch;
+  s.capacity = capacity;
+  s.k_cache = (bf16*)k_cache;
+  s.v_cache = (bf16*)v_cache;
+  s.len_upper.assign(kv_len, kv_len + batch);
+  s.max_rows = batch * (kMaxK + 1);
+  const size_t R = s.max_rows, H = m.cfg.hidden, F = m.cfg.ffn;
+  size_t bytes = 4096 + 3 * align_up((size_t)(batch + 1) * 4, 256);
+  bytes += align_up(R * H * 4, 256) + align_up(R * H * 2, 256) +
+           align_up(R * m.qkv_rows * 4, 256) + align_up(R * m.q_dim * 4, 256) +
+           align_up(R * m.q_dim * 2, 256) + align_up(R * F * 2, 256) + align_up(R * 8, 256);
+  cudaError_t e = cudaMalloc(&s.work, bytes);
+  if (e != cudaSuccess) {
+    delete kh;
+    return fail(AS2D_ERR_CUDA, std::string("cudaMalloc of the working memory: ") + cudaGetErrorString(e));
+  }
+  s.work_bytes = bytes;
+  Carver cv{(char*)s.work};
+  s.d_len = cv.take<int32_t>(batch);
+  s.d_root = cv.take<int32_t>(batch);
+  s.d_err = cv.take<int32_t>(batch + 1);
+  s.h = cv.take<float>(R * H);
+  s.xn = cv.take<bf16>(R * H);
+  s.qkv = cv.take<float>(R * m.qkv_rows);
+  s.q = cv.take<float>(R * m.q_dim);
+  s.ao = cv.take<bf16>(R * m.q_dim);
+  s.u = cv.take<bf16>(R * F);
+  s.best = cv.take<unsigned long long>(R);
+  e = cudaMemset(s.work, 0, bytes);
+  if (e == cudaSuccess) e = cudaMemcpy(s.d_len, kv_len, batch * 4, cudaMemcpyHostToDevice);
+  if (e == cudaSuccess) e = cudaMemcpy(s.d_root, root_tokens, batch * 4, cudaMemcpyHostToDevice);
+  if (e == cudaSuccess) e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) {
+    cudaFree(s.work);
+    delete kh;
+    return fail(AS2D_ERR_CUDA, std::string("initialising the state: ") + cudaGetErrorString(e));
+  }
+  *out = kh;
+  return AS2D_OK;
+}
+
+extern "C" void as2d_kv_free(as2d_kv* kh) {
+  if (!kh) return;
+  for (cudaEvent_t e : kh->s.prof_events) cudaEventDestroy(e);
+  cudaFree(kh->s.work);
+  delete kh;
+}
+
+namespace {
+
+// Event pair around the launches of one kernel class in one layer, recorded
+// only while that class is being profiled.
+struct ProfScope {
+  KvState& s;
+  cudaStream_t st;
+  bool on;
+  int idx = -1;
+  ProfScope(KvState& s_, int cls, cudaStream_t st_) : s(s_), st(st_), on(s_.prof_class == cls) {
+    if (!on) return;
+    if ((size_t)(2 * s.prof_used + 2) > s.prof_events.size()) {
+      for (int i = 0; i < 64; ++i) {
+        cudaEvent_t e;
+        if (cudaEventCreate(&e) != cudaSuccess) { on = false; return; }
+        s.prof_events.push_back(e);
+      }
+    }
+    idx = s.prof_used++;
+    cudaEventRecord(s.prof_events[2 * idx], st);
+  }
+  ~ProfScope() {
+    if (on && idx >= 0) cudaEventRecord(s.prof_events[2 * idx + 1], st);
+  }
+};
+
+#define LAUNCH(cls, expr)                        \
+  do {                                           \
+    ProfScope ps_(s, cls, st);                   \
+    CUDA_TRY(expr);                              \
+    ++s.launches;                                \
+  } while (0)
+
+as2d_status run_block(KvState& s, const int32_t* cand, const int32_t* k,
+                      const as2d_verify_out* out, cudaStream_t st) {
+  if (!out || !out->n_accepted || !out->correction_token)
+    return fail(AS2D_ERR_INVALID_ARG, "out, out->n_accepted and out->correction_token are required");
+  RowMap rm;
+  rm.batch = s.batch;
+  rm.start[0] = 0;
+  int total_k = 0;
+  for (int b = 0; b < s.batch; ++b) {
+    const int kb = k ? k[b] : 0;
+    if (kb < 0 || kb > kMaxK)
+      return fail(AS2D_ERR_INVALID_ARG, "k must be in [0, AS2D_MAX_K]");
+    if (s.len_upper[b] + kb + 1 > s.capacity)
+      return fail(AS2D_ERR_CAPACITY, "length bound + k + 1 exceeds the cache capacity");
+    rm.start[b + 1] = rm.start[b] + kb + 1;
+    total_k += kb;
+  }
+  rm.rows = rm.start[s.batch];
+  if (total_k > 0 && !cand) return fail(AS2D_ERR_INVALID_ARG, "candidates is NULL");
+  const Model& m = *s.model;
+  const as2d_config& c = m.cfg;
+
+  LAUNCH(AS2D_KERNEL_OTHER, launch_embed(rm, m, s, cand, st));
+  for (int l = 0; l < c.n_layers; ++l) {
+    {
+      ProfScope ps(s, AS2D_KERNEL_QKV, st);
+      LAUNCH(-1, launch_rmsnorm(rm, m, s, m.attn_norm[l], st));
+      LAUNCH(-1, launch_gemv_qkv(rm, m, s, l, st));
+    }
+    {
+      ProfScope ps(s, AS2D_KERNEL_ATTENTION, st);
+      LAUNCH(-1, launch_rope_append(rm, m, s, l, st));
+      LAUNCH(-1, launch_attention(rm, m, s, l, st));
+    }
+    LAUNCH(AS2D_KERNEL_O, launch_gemv_o(rm, m, s, l, st));
+    {
+      ProfScope ps(s, AS2D_KERNEL_GATE_UP, st);
+      LAUNCH(-1, launch_rmsnorm(rm, m, s, m.mlp_norm[l], st));
+      LAUNCH(-1, launch_gemv_gate_up(rm, m, s, l, st));
+    }
+    LAUNCH(AS2D_KERNEL_DOWN, launch_gemv_down(rm, m, s, l, st));
+  }
+  {
+    ProfScope ps(s, AS2D_KERNEL_LM_HEAD, st);
+    LAUNCH(-1, launch_rmsnorm(rm, m, s, m.final_norm, st));
+    LAUNCH(-1, launch_lm_head(rm, m, s, out->logits, st));
+  }
+  LAUNCH(AS2D_KERNEL_OTHER, launch_accept(rm, m, s, cand, *out, st));
+  for (int b = 0; b < s.batch; ++b) s.len_upper[b] += (k ? k[b] : 0) + 1;
+  return AS2D_OK;
+}
+
+}  // namespace
+
+extern "C" as2d_status as2d_verify_block(as2d_kv* kh, const int32_t* candidates,
+                                         const int32_t* k,
+                                         const as2d_verify_out* out,
+                                         void* stream) {
+  g_err.clear();
+  if (!kh || !k) return fail(AS2D_ERR_INVALID_ARG, "kv and k are required");
+  return run_block(kh->s, candidates, k, out, (cudaStream_t)stream);
+}
+
+extern "C" as2d_status as2d_decode_step(as2d_kv* kh, const as2d_verify_out* out,
+                                        void* stream) {
+  g_err.clear();
+  if (!kh) return fail(AS2D_ERR_INVALID_ARG, "kv is NULL");
+  return run_block(kh->s, nullptr, nullptr, out, (cudaStream_t)stream);
+}
+
+extern "C" as2d_status as2d_kv_rollback(as2d_kv* kh, const int32_t* new_len,
+                                        const int32_t* new_root, void* stream) {
+  g_err.clear();
+  if (!kh || !new_len || !new_root)
+    return fail(AS2D_ERR_INVALID_ARG, "kv, new_len and new_root are required");
+  KvState& s = kh->s;
+  for (int b = 0; b < s.batch; ++b) {
+    if (new_len[b] < 0 || new_len[b] >= s.capacity)
+      return fail(AS2D_ERR_INVALID_ARG, "new_len must be in [0, capacity)");
+    if (new_root[b] < 0 || new_root[b] >= s.model->cfg.vocab)
+      return fail(AS2D_ERR_INVALID_ARG, "new_root outside [0, vocab)");
+  }
+  CUDA_TRY(launch_rollback(s, new_len, new_root, (cudaStream_t)stream));
+  for (int b = 0; b < s.batch; ++b) s.len_upper[b] = new_len[b];
+  return AS2D_OK;
+}
+
+extern "C" as2d_status as2d_kv_read_state(as2d_kv* kh, int32_t* len,
+                                          int32_t* root, void* stream) {
+  g_err.clear();
+  if (!kh) return fail(AS2D_ERR_INVALID_ARG, "kv is NULL");
+  KvState& s = kh->s;
+  CUDA_TRY(cudaStreamSynchronize((cudaStream_t)stream));
+  int32_t tmp_len[kMaxBatch], tmp_root[kMaxBatch];
+  CUDA_TRY(cudaMemcpy(tmp_len, s.d_len, s.batch * 4, cudaMemcpyDeviceToHost));
+  CUDA_TRY(cudaMemcpy(tmp_root, s.d_root, s.batch * 4, cudaMemcpyDeviceToHost));
+  for (int b = 0; b < s.batch; ++b) {
+    s.len_upper[b] = tmp_len[b];
+    if (len) len[b] = tmp_len[b];
+    if (root) root[b] = tmp_root[b];
+  }
+  return AS2D_OK;
+}
+
+extern "C" as2d_status as2d_kv_device_state(as2d_kv* kh, const int32_t** len,
+                                            const int32_t** root) {
+  g_err.clear();
+  if (!kh) return fail(AS2D_ERR_INVALID_ARG, "kv is NULL");
+  if (len) *len = kh->s.d_len;
+  if (root) *root = kh->s.d_root;
+  return AS2D_OK;
+}
+
+extern "C" as2d_status as2d_kv_check(as2d_kv* kh, void* stream) {
+  g_err.clear();
+  if (!kh) return fail(AS2D_ERR_INVALID_ARG, "kv is NULL");
+  CUDA_TRY(cudaStreamSynchronize((cudaStream_t)stream));
+  int32_t err = 0;
+  CUDA_TRY(cudaMemcpy(&err, kh->s.d_err, 4, cudaMemcpyDeviceToHost));
+  if (err != 0) {
+    int32_t zero = 0;
+    CUDA_TRY(cudaMemcpy(kh->s.d_err, &zero, 4, cudaMemcpyHostToDevice));
+    std::string msg = "device error:";
+    if (err & kErrBadToken) msg += " candidate or root token outside [0, vocab);";
+    if (err & kErrRollback) msg += " rollback beyond the committed length;";
+    if (err & kErrTimeout) msg += " a kernel wait timed out;";
+    return fail(AS2D_ERR_DEVICE, msg);
+  }
+  return AS2D_OK;
+}
+
+extern "C" as2d_status as2d_kv_profile(as2d_kv* kh, int32_t kernel_class) {
+  g_err.clear();
+  if (!kh) return fail(AS2D_ERR_INVALID_ARG, "kv is NULL");
+  if (kernel_class < -1 || kernel_class >= AS2D_KERNEL_CLASSES)
+    return fail(AS2D_ERR_INVALID_ARG, "kernel_class must be -1 or a class id");
+  kh->s.prof_class = kernel_class;
+  return AS2D_OK;
+}
+
+extern "C" as2d_status as2d_kv_profile_read(as2d_kv* kh, int32_t* launches,
+                                            double* total_ms,
+                                            int64_t* all_launches) {
+  g_err.clear();
+  if (!kh) return fail(AS2D_ERR_INVALID_ARG, "kv is NULL");
+  KvState& s = kh->s;
+  double tot = 0.0;
+  for (int i = 0; i < s.prof_used; ++i) {
+    CUDA_TRY(cudaEventSynchronize(s.prof_events[2 * i + 1]));
+    float ms = 0.f;
+    CUDA_TRY(cudaEventElapsedTime(&ms, s.prof_events[2 * i], s.prof_events[2 * i + 1]));
+    tot += ms;
+  }
+  if (launches) *launches = s.prof_used;
+  if (total_ms) *total_ms = tot;
+  if (all_launches) *all_launches = s.launches;
+  s.prof_used = 0;
+  s.launches = 0;
+  return AS2D_OK;
+}
