@@ -227,6 +227,21 @@ def run_ours(args, ws, rank, local):
         committed = int((n_np + 1).sum())
         plan_match = float(np.mean(n_np == plans[:, 0]))
 
+        # per-class device time per block (diagnostic, after the timed region)
+        breakdown = {}
+        for cls_name in ("qkv", "attention", "o", "gate_up", "down", "lm_head", "other"):
+            state.rollback([L0], [root0], sh)
+            state.read_state(sh)
+            state.profile(cls_name)
+            state.profile_read()
+            nb_blocks = min(8, steps)
+            for i in range(nb_blocks):
+                block(i, i)
+            n_cls, ms_cls, _ = state.profile_read()
+            breakdown[cls_name] = round(ms_cls / nb_blocks * 1e3, 1)
+        state.profile(None)
+        state.check(sh)
+
         e2e = None
         if not args.no_e2e:
             e2e = run_e2e(args, lib, W, state, traj, plans, cfg, L0, root0, sh, stream)
@@ -286,6 +301,7 @@ def run_ours(args, ws, rank, local):
         "step_roofline": step_roof,
         "roofline": roofline,
         "gpu_launches": int(all_launches),
+        "class_us_per_block": breakdown,
         "clocks": clk,
         "e2e": e2e,
     }

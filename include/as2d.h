@@ -117,7 +117,8 @@ as2d_status as2d_model_load(const as2d_config* cfg, const as2d_weights* w,
    entries of forwarded rows; the caller keeps both buffers alive until
    as2d_kv_free.  kv_len, root_tokens: host int32 [batch]; root_tokens[b] is
    request b's pending known root (the first token chosen after prefill).
-   Allocates the state's device working memory.  Synchronises the device. */
+   capacity <= 65536 (AS2D_ERR_UNSUPPORTED above).  Allocates the state's
+   device working memory.  Synchronises the device. */
 as2d_status as2d_kv_init_prefilled(as2d_model* model, int32_t batch,
                                    const int32_t* kv_len, int32_t capacity,
                                    void* k_cache, void* v_cache,

@@ -32,7 +32,8 @@ def headers():
 
 def _compile(src, verbose_ptxas=False):
     obj = os.path.join(OBJ_DIR, os.path.basename(src) + ".o")
-    cmd = [NVCC, *ARCH, *CFLAGS, "-c", src, "-o", obj]
+    extra = os.environ.get("AS2D_NVCC_EXTRA", "").split()  # tuning experiments only
+    cmd = [NVCC, *ARCH, *CFLAGS, *extra, "-c", src, "-o", obj]
     if verbose_ptxas:
         cmd += ["-Xptxas", "-v"]
     r = subprocess.run(cmd, capture_output=True, text=True)

@@ -1,6 +1,7 @@
 // as2d_api.cu -- the C-ABI of include/as2d.h: argument checking, ownership,
 // weight re-layout at load time, and the per-call launch sequence of the
 // verification pass (Section 3.2; App. C.2).
+#include <cstdlib>
 #include <cstring>
 #include <string>
 
@@ -46,6 +47,39 @@ struct Carver {
     return p;
   }
 };
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = (EncodeTiledFn)ptr;
+  }
+  return fn;
+}
+
+// Row-major bf16 matrix [outer][inner] viewed by TMA in boxes of
+// box_inner x box_outer elements with 128-byte swizzling.
+bool encode_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer,
+               uint32_t box_inner, uint32_t box_outer) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {inner * 2};
+  cuuint32_t box[2] = {box_inner, box_outer};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
 
 as2d_status check_config(const as2d_config* c) {
   if (!c) return fail(AS2D_ERR_INVALID_ARG, "config is NULL");
@@ -101,14 +135,16 @@ extern "C" as2d_status as2d_model_load(const as2d_config* cfg,
   cudaDeviceGetAttribute(&m.sm_count, cudaDevAttrMultiProcessorCount, dev);
   (void)d;
 
-  const size_t per_layer_bf16 = (size_t)m.qkv_rows * H + H * m.q_dim + 2 * F * H + H * F;
-  size_t bytes = 0;
-  bytes += align_up(V * H * 2, 256) * 2;
-  bytes += L * (align_up((size_t)m.qkv_rows * H * 2, 256) + align_up(H * m.q_dim * 2, 256) +
-                align_up(2 * F * H * 2, 256) + align_up(H * F * 2, 256) +
+  const size_t qkv_packed = packed_elems(m.qkv_rows, (int)H);
+  const size_t o_packed = packed_elems((int)H, m.q_dim);
+  const size_t gu_packed = packed_elems((int)(2 * F), (int)H);
+  const size_t down_packed = packed_elems((int)H, (int)F);
+  const size_t lm_packed = packed_elems((int)V, (int)H);
+  size_t bytes = align_up(V * H * 2, 256) + align_up(lm_packed * 2, 256);
+  bytes += L * (align_up(qkv_packed * 2, 256) + align_up(o_packed * 2, 256) +
+                align_up(gu_packed * 2, 256) + align_up(down_packed * 2, 256) +
                 2 * align_up(H * 4, 256));
   bytes += align_up(H * 4, 256) + 4096;
-  (void)per_layer_bf16;
   cudaError_t e = cudaMalloc(&m.arena, bytes);
   if (e != cudaSuccess) {
     delete mh;
@@ -129,33 +165,45 @@ extern "C" as2d_status as2d_model_load(const as2d_config* cfg,
   } while (0)
 
   bf16* embed = cv.take<bf16>(V * H);
-  bf16* lm = cv.take<bf16>(V * H);
+  bf16* lm = cv.take<bf16>(lm_packed);
   float* fnorm = cv.take<float>(H);
   LOAD_TRY(cudaMemcpy(embed, w->embed, V * H * 2, cudaMemcpyDeviceToDevice));
-  LOAD_TRY(cudaMemcpy(lm, w->lm_head, V * H * 2, cudaMemcpyDeviceToDevice));
+  {
+    const void* segs[1] = {w->lm_head};
+    const int rows[1] = {(int)V};
+    LOAD_TRY(pack_weights(lm, (int)V, (int)H, segs, rows, 1, false, 0));
+  }
   LOAD_TRY(launch_f32_from_bf16(fnorm, w->final_norm, H, 0));
   m.embed = embed;
   m.lm_head = lm;
   m.final_norm = fnorm;
   for (int l = 0; l < L; ++l) {
-    bf16* qkv = cv.take<bf16>((size_t)m.qkv_rows * H);
-    bf16* wo = cv.take<bf16>(H * m.q_dim);
-    bf16* gu = cv.take<bf16>(2 * F * H);
-    bf16* wd = cv.take<bf16>(H * F);
+    bf16* qkv = cv.take<bf16>(qkv_packed);
+    bf16* wo = cv.take<bf16>(o_packed);
+    bf16* gu = cv.take<bf16>(gu_packed);
+    bf16* wd = cv.take<bf16>(down_packed);
     float* an = cv.take<float>(H);
     float* mn = cv.take<float>(H);
-    LOAD_TRY(cudaMemcpy(qkv, w->w_q[l], (size_t)m.q_dim * H * 2, cudaMemcpyDeviceToDevice));
-    LOAD_TRY(cudaMemcpy(qkv + (size_t)m.q_dim * H, w->w_k[l], (size_t)m.kv_dim * H * 2,
-                        cudaMemcpyDeviceToDevice));
-    LOAD_TRY(cudaMemcpy(qkv + (size_t)(m.q_dim + m.kv_dim) * H, w->w_v[l],
-                        (size_t)m.kv_dim * H * 2, cudaMemcpyDeviceToDevice));
-    LOAD_TRY(cudaMemcpy(wo, w->w_o[l], H * m.q_dim * 2, cudaMemcpyDeviceToDevice));
-    // gate/up interleaved in blocks of 64 rows: [64 gate | 64 up] per 128 rows
-    LOAD_TRY(cudaMemcpy2D(gu, 128 * H * 2, w->w_gate[l], 64 * H * 2, 64 * H * 2, F / 64,
-                          cudaMemcpyDeviceToDevice));
-    LOAD_TRY(cudaMemcpy2D(gu + 64 * H, 128 * H * 2, w->w_up[l], 64 * H * 2, 64 * H * 2, F / 64,
-                          cudaMemcpyDeviceToDevice));
-    LOAD_TRY(cudaMemcpy(wd, w->w_down[l], H * F * 2, cudaMemcpyDeviceToDevice));
+    {
+      const void* segs[3] = {w->w_q[l], w->w_k[l], w->w_v[l]};
+      const int rows[3] = {m.q_dim, m.kv_dim, m.kv_dim};
+      LOAD_TRY(pack_weights(qkv, m.qkv_rows, (int)H, segs, rows, 3, false, 0));
+    }
+    {
+      const void* segs[1] = {w->w_o[l]};
+      const int rows[1] = {(int)H};
+      LOAD_TRY(pack_weights(wo, (int)H, m.q_dim, segs, rows, 1, false, 0));
+    }
+    {
+      const void* segs[2] = {w->w_gate[l], w->w_up[l]};
+      const int rows[2] = {(int)F, (int)F};
+      LOAD_TRY(pack_weights(gu, (int)(2 * F), (int)H, segs, rows, 2, true, 0));
+    }
+    {
+      const void* segs[1] = {w->w_down[l]};
+      const int rows[1] = {(int)H};
+      LOAD_TRY(pack_weights(wd, (int)H, (int)F, segs, rows, 1, false, 0));
+    }
     LOAD_TRY(launch_f32_from_bf16(an, w->attn_norm[l], H, 0));
     LOAD_TRY(launch_f32_from_bf16(mn, w->mlp_norm[l], H, 0));
     m.w_qkv.push_back(qkv);
@@ -189,6 +237,8 @@ extern "C" as2d_status as2d_kv_init_prefilled(as2d_model* mh, int32_t batch,
   if (batch < 1 || batch > kMaxBatch)
     return fail(AS2D_ERR_INVALID_ARG, "batch must be in [1, AS2D_MAX_BATCH]");
   if (capacity < 1) return fail(AS2D_ERR_INVALID_ARG, "capacity must be positive");
+  if (capacity > 65536)
+    return fail(AS2D_ERR_UNSUPPORTED, "capacity above 65536 positions is not supported");
   const Model& m = mh->m;
   for (int b = 0; b < batch; ++b) {
     if (kv_len[b] < 0 || kv_len[b] >= capacity)
@@ -205,11 +255,21 @@ extern "C" as2d_status as2d_kv_init_prefilled(as2d_model* mh, int32_t batch,
   s.v_cache = (bf16*)v_cache;
   s.len_upper.assign(kv_len, kv_len + batch);
   s.max_rows = batch * (kMaxK + 1);
-  const size_t R = s.max_rows, H = m.cfg.hidden, F = m.cfg.ffn;
+  s.nb_max = nb_for_rows(s.max_rows);
+  s.rows_alloc = s.max_rows > s.nb_max ? s.max_rows : s.nb_max;
+  const size_t R = s.rows_alloc, H = m.cfg.hidden, F = m.cfg.ffn;
+  const size_t max_tiles = ((size_t)(m.cfg.vocab > 2 * F ? m.cfg.vocab : 2 * F) + 127) / 128 + 64;
   size_t bytes = 4096 + 3 * align_up((size_t)(batch + 1) * 4, 256);
   bytes += align_up(R * H * 4, 256) + align_up(R * H * 2, 256) +
-           align_up(R * m.qkv_rows * 4, 256) + align_up(R * m.q_dim * 4, 256) +
-           align_up(R * m.q_dim * 2, 256) + align_up(R * F * 2, 256) + align_up(R * 8, 256);
+           align_up(R * m.q_dim * 4, 256) +
+           align_up(R * m.q_dim * 2, 256) + align_up(R * F * 2, 256) + align_up(R * 8, 256) +
+           align_up(R * (m.cfg.head_dim / 2) * 8, 256) + align_up(R * (H / 128) * 4, 256) +
+           align_up((size_t)m.sm_count * 2 * s.nb_max * 128 * 4, 256) + align_up(max_tiles * 4, 256);
+  const int group = m.cfg.n_q_heads / m.cfg.n_kv_heads;
+  s.attn_parts = attn_partitions(capacity);
+  s.attn_qmax = ((kMaxK + 1) * group + 15) / 16 * 16;
+  const size_t attn_rows = (size_t)batch * m.cfg.n_kv_heads * s.attn_parts * s.attn_qmax;
+  bytes += align_up(attn_rows * m.cfg.head_dim * 4, 256) + align_up(attn_rows * 8, 256);
   cudaError_t e = cudaMalloc(&s.work, bytes);
   if (e != cudaSuccess) {
     delete kh;
@@ -222,11 +282,29 @@ extern "C" as2d_status as2d_kv_init_prefilled(as2d_model* mh, int32_t batch,
   s.d_err = cv.take<int32_t>(batch + 1);
   s.h = cv.take<float>(R * H);
   s.xn = cv.take<bf16>(R * H);
-  s.qkv = cv.take<float>(R * m.qkv_rows);
   s.q = cv.take<float>(R * m.q_dim);
   s.ao = cv.take<bf16>(R * m.q_dim);
   s.u = cv.take<bf16>(R * F);
   s.best = cv.take<unsigned long long>(R);
+  s.rope = cv.take<float2>(R * (m.cfg.head_dim / 2));
+  s.ss = cv.take<float>(R * (H / 128));
+  s.ws = cv.take<float>((size_t)m.sm_count * 2 * s.nb_max * 128);
+  s.counters = cv.take<int>(max_tiles);
+  s.attn_o = cv.take<float>(attn_rows * m.cfg.head_dim);
+  s.attn_ml = cv.take<float2>(attn_rows);
+  bool ok = true;
+  for (int i = 0; i < kNbCount && ok; ++i) {
+    const int nb = 16 << i;
+    if (nb > s.nb_max) break;
+    ok = encode_2d(&s.tm_xn[i], s.xn, H, R, 64, nb) &&
+         encode_2d(&s.tm_ao[i], s.ao, m.q_dim, R, 64, nb) &&
+         encode_2d(&s.tm_u[i], s.u, F, R, 64, nb);
+  }
+  if (!ok) {
+    cudaFree(s.work);
+    delete kh;
+    return fail(AS2D_ERR_CUDA, "cuTensorMapEncodeTiled failed for an activation buffer");
+  }
   e = cudaMemset(s.work, 0, bytes);
   if (e == cudaSuccess) e = cudaMemcpy(s.d_len, kv_len, batch * 4, cudaMemcpyHostToDevice);
   if (e == cudaSuccess) e = cudaMemcpy(s.d_root, root_tokens, batch * 4, cudaMemcpyHostToDevice);
@@ -280,6 +358,38 @@ struct ProfScope {
     ++s.launches;                                \
   } while (0)
 
+// One projection on the tensor cores: row chunks of at most 256 token rows.
+cudaError_t tc_project(int epi, const Model& m, KvState& s, const RowMap& rm, const bf16* w,
+                       const CUtensorMap* xmaps, int N, int K, TcParams p, cudaStream_t st) {
+  p.w = w;
+  p.N = N;
+  p.K = K;
+  p.n_tiles = (N + 127) / 128;
+  p.kb = (K + 63) / 64;
+  p.units = (long long)p.n_tiles * p.kb;
+  p.grid = (int)(p.units < m.sm_count ? p.units : m.sm_count);
+  p.ws = s.ws;
+  p.counters = s.counters;
+  p.err = s.d_err;
+  p.timeout_ns = 2000000000ull;
+  p.rm = rm;
+  for (int row0 = 0; row0 < rm.rows; row0 += 256) {
+    p.row0 = row0;
+    p.rows = rm.rows - row0 < 256 ? rm.rows - row0 : 256;
+    const int nb = nb_for_rows(p.rows);
+    const CUtensorMap& x = xmaps[nb_index(nb)];
+    cudaError_t e;
+    switch (epi) {
+      case TC_QKV: e = tc_gemm_qkv(nb, x, p, st); break;
+      case TC_RESID: e = tc_gemm_resid(nb, x, p, st); break;
+      case TC_SWIGLU: e = tc_gemm_swiglu(nb, x, p, st); break;
+      default: e = tc_gemm_logits(nb, x, p, st); break;
+    }
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
 as2d_status run_block(KvState& s, const int32_t* cand, const int32_t* k,
                       const as2d_verify_out* out, cudaStream_t st) {
   if (!out || !out->n_accepted || !out->correction_token)
@@ -302,31 +412,43 @@ as2d_status run_block(KvState& s, const int32_t* cand, const int32_t* k,
   const Model& m = *s.model;
   const as2d_config& c = m.cfg;
 
+  // One pass of the verification step (Section 3.2; App. C.2): embedding
+  // gather, n_layers x {QKV + RoPE + KV append, attention, O + residual,
+  // gate/up + SwiGLU, down + residual}, LM head + argmax, accept scan.
   LAUNCH(AS2D_KERNEL_OTHER, launch_embed(rm, m, s, cand, st));
+  TcParams tp{};
+  tp.h = s.h;
+  tp.u = s.u;
+  tp.q = s.q;
+  tp.kc = s.k_cache;
+  tp.vc = s.v_cache;
+  tp.rope = s.rope;
+  tp.len = s.d_len;
+  tp.batch = s.batch;
+  tp.cap = s.capacity;
+  tp.nq = c.n_q_heads;
+  tp.nkv = c.n_kv_heads;
+  tp.d = c.head_dim;
+  tp.logits = out->logits;
+  tp.best = s.best;
+  tp.xn = s.xn;
+  tp.ss = s.ss;
+  tp.ss_ld = s.rows_alloc;
+  tp.n_htiles = c.hidden / 128;
+  tp.eps = c.rms_eps;
+  tp.hidden = c.hidden;
+  const int H = c.hidden, F = c.ffn;
   for (int l = 0; l < c.n_layers; ++l) {
-    {
-      ProfScope ps(s, AS2D_KERNEL_QKV, st);
-      LAUNCH(-1, launch_rmsnorm(rm, m, s, m.attn_norm[l], st));
-      LAUNCH(-1, launch_gemv_qkv(rm, m, s, l, st));
-    }
-    {
-      ProfScope ps(s, AS2D_KERNEL_ATTENTION, st);
-      LAUNCH(-1, launch_rope_append(rm, m, s, l, st));
-      LAUNCH(-1, launch_attention(rm, m, s, l, st));
-    }
-    LAUNCH(AS2D_KERNEL_O, launch_gemv_o(rm, m, s, l, st));
-    {
-      ProfScope ps(s, AS2D_KERNEL_GATE_UP, st);
-      LAUNCH(-1, launch_rmsnorm(rm, m, s, m.mlp_norm[l], st));
-      LAUNCH(-1, launch_gemv_gate_up(rm, m, s, l, st));
-    }
-    LAUNCH(AS2D_KERNEL_DOWN, launch_gemv_down(rm, m, s, l, st));
+    tp.layer = l;
+    LAUNCH(AS2D_KERNEL_QKV, tc_project(TC_QKV, m, s, rm, m.w_qkv[l], s.tm_xn, m.qkv_rows, H, tp, st));
+    LAUNCH(AS2D_KERNEL_ATTENTION, launch_attention_split(rm, m, s, l, st));
+    tp.g_next = m.mlp_norm[l];
+    LAUNCH(AS2D_KERNEL_O, tc_project(TC_RESID, m, s, rm, m.w_o[l], s.tm_ao, H, m.q_dim, tp, st));
+    LAUNCH(AS2D_KERNEL_GATE_UP, tc_project(TC_SWIGLU, m, s, rm, m.w_gu[l], s.tm_xn, 2 * F, H, tp, st));
+    tp.g_next = (l + 1 < c.n_layers) ? m.attn_norm[l + 1] : m.final_norm;
+    LAUNCH(AS2D_KERNEL_DOWN, tc_project(TC_RESID, m, s, rm, m.w_down[l], s.tm_u, H, F, tp, st));
   }
-  {
-    ProfScope ps(s, AS2D_KERNEL_LM_HEAD, st);
-    LAUNCH(-1, launch_rmsnorm(rm, m, s, m.final_norm, st));
-    LAUNCH(-1, launch_lm_head(rm, m, s, out->logits, st));
-  }
+  LAUNCH(AS2D_KERNEL_LM_HEAD, tc_project(TC_LOGITS, m, s, rm, m.lm_head, s.tm_xn, c.vocab, H, tp, st));
   LAUNCH(AS2D_KERNEL_OTHER, launch_accept(rm, m, s, cand, *out, st));
   for (int b = 0; b < s.batch; ++b) s.len_upper[b] += (k ? k[b] : 0) + 1;
   return AS2D_OK;

@@ -42,6 +42,64 @@ enum : int32_t {
   kErrTimeout = 4,
 };
 
+enum TcEpi { TC_QKV = 0, TC_RESID = 1, TC_SWIGLU = 2, TC_LOGITS = 3 };
+
+struct TcParams {
+  const bf16* w;         // packed weight blocks (k_pack.cu), unit u at u * 8192
+  int N, K;              // logical W is [N][K]
+  int n_tiles, kb;       // 128-row tiles, 64-column k-blocks
+  long long units;       // n_tiles * kb
+  int grid;              // CTAs (persistent)
+  int rows;              // token rows handled by this launch
+  int row0;              // first token row of this launch
+  float* ws;             // [grid][2][NB][128] partial tiles
+  int* counters;         // [n_tiles] arrivals; zero between launches
+  int* err;
+  unsigned long long timeout_ns;
+  // epilogue operands
+  float* h;              // RESID: h[m][n] += D (ld = N)
+  bf16* u;               // SWIGLU: u[m][j], ld = N / 2
+  float* q;              // QKV: rotated queries [m][nq * d]
+  bf16* kc;
+  bf16* vc;
+  const float2* rope;    // [m][d / 2] (cos, sin) of the row's position
+  const int32_t* len;
+  int layer, batch, cap, nq, nkv, d;
+  float* logits;         // LOGITS (nullable), ld = N
+  unsigned long long* best;
+  // RMSNorm folded into the GEMMs: a RESID epilogue leaves, for the next
+  // projection, xn = bf16(h * g_next) and per-128-column sums of h^2; the
+  // next projection scales its accumulator by 1 / rms of its row.
+  const float* g_next;   // RESID: gain of the norm that consumes h next
+  bf16* xn;              // RESID: [rows][N] next operand
+  float* ss;             // [N / 128][rows_alloc] partial sums of squares
+  int ss_ld;             // rows_alloc
+  int n_htiles;          // hidden / 128 (consumer side)
+  float eps;
+  int hidden;
+  RowMap rm;
+};
+
+// Launch with programmatic stream serialization: the kernel may be scheduled
+// while its predecessor in the stream is still running; every kernel of the
+// library calls griddepcontrol.wait before it touches memory that an earlier
+// kernel of the stream wrote.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t st, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, args...);
+}
+
 struct Model {
   as2d_config cfg;
   int qkv_rows;      // (n_q + 2 n_kv) * head_dim
@@ -51,14 +109,23 @@ struct Model {
   void* arena = nullptr;  // every weight below lives here
   size_t arena_bytes = 0;
   const bf16* embed = nullptr;    // [V][H]
-  const bf16* lm_head = nullptr;  // [V][H]
+  const bf16* lm_head = nullptr;  // logical [V][H], packed tile-major
   const float* final_norm = nullptr;
-  std::vector<const bf16*> w_qkv;   // [(nq + 2 nkv) d][H]: q rows, k rows, v rows
-  std::vector<const bf16*> w_o;     // [H][nq d]
-  std::vector<const bf16*> w_gu;    // [2F][H]: blocks of 64 gate rows, 64 up rows
-  std::vector<const bf16*> w_down;  // [H][F]
+  // projection weights, packed tile-major (k_pack.cu)
+  std::vector<const bf16*> w_qkv;   // logical [(nq + 2 nkv) d][H]: q rows, k rows, v rows
+  std::vector<const bf16*> w_o;     // logical [H][nq d]
+  std::vector<const bf16*> w_gu;    // logical [2F][H]: per 128 rows, 64 gate then 64 up
+  std::vector<const bf16*> w_down;  // logical [H][F]
   std::vector<const float*> attn_norm, mlp_norm;  // fp32 gains [H]
 };
+
+constexpr int kNbCount = 5;  // token-row paddings 16, 32, 64, 128, 256
+inline int nb_index(int nb) { return nb == 16 ? 0 : nb == 32 ? 1 : nb == 64 ? 2 : nb == 128 ? 3 : 4; }
+inline int nb_for_rows(int rows) {
+  int nb = 16;
+  while (nb < rows && nb < 256) nb <<= 1;
+  return nb;
+}
 
 struct KvState {
   Model* model = nullptr;
@@ -77,11 +144,22 @@ struct KvState {
   size_t work_bytes = 0;
   float* h = nullptr;        // [rows][H] residual stream, fp32
   bf16* xn = nullptr;        // [rows][H] normalised activations
-  float* qkv = nullptr;      // [rows][qkv_rows]
   float* q = nullptr;        // [rows][nq][d] rotated queries
   bf16* ao = nullptr;        // [rows][nq d] attention output
   bf16* u = nullptr;         // [rows][F] SwiGLU output
   unsigned long long* best = nullptr;  // [rows] packed (logit, index) maxima
+  float2* rope = nullptr;    // [rows][d/2] (cos, sin) at each row's position
+  int rows_alloc = 0;        // activation rows allocated (>= every NB used)
+  int nb_max = 16;
+  float* ws = nullptr;       // [sm_count][2][nb_max][128] partial GEMM tiles
+  int* counters = nullptr;   // [max tiles] stream-K arrival counters
+  float* ss = nullptr;       // [hidden / 128][rows_alloc] partial sums of h^2
+  float* attn_o = nullptr;   // [batch][n_kv][parts][qmax][d] attention partials
+  float2* attn_ml = nullptr; // [batch][n_kv][parts][qmax] (max, sum) base 2
+  int attn_parts = 0;        // 64-key partitions of the capacity
+  int attn_qmax = 0;         // (kMaxK + 1) * group, rounded up to 16
+  // TMA descriptors of the activation operands, per token-row padding
+  CUtensorMap tm_xn[kNbCount], tm_ao[kNbCount], tm_u[kNbCount];
   // measurement support
   int prof_class = -1;
   std::vector<cudaEvent_t> prof_events;  // pairs
@@ -92,27 +170,31 @@ struct KvState {
 // Launchers (k_basic.cu).  All enqueue on `st` and return cudaGetLastError().
 cudaError_t launch_embed(const RowMap& m, const Model& md, KvState& kv,
                          const int32_t* cand, cudaStream_t st);
-cudaError_t launch_rmsnorm(const RowMap& m, const Model& md, KvState& kv,
-                           const float* gain, cudaStream_t st);
-cudaError_t launch_gemv_qkv(const RowMap& m, const Model& md, KvState& kv,
-                            int layer, cudaStream_t st);
-cudaError_t launch_rope_append(const RowMap& m, const Model& md, KvState& kv,
-                               int layer, cudaStream_t st);
-cudaError_t launch_attention(const RowMap& m, const Model& md, KvState& kv,
-                             int layer, cudaStream_t st);
-cudaError_t launch_gemv_o(const RowMap& m, const Model& md, KvState& kv,
-                          int layer, cudaStream_t st);
-cudaError_t launch_gemv_gate_up(const RowMap& m, const Model& md, KvState& kv,
-                                int layer, cudaStream_t st);
-cudaError_t launch_gemv_down(const RowMap& m, const Model& md, KvState& kv,
-                             int layer, cudaStream_t st);
-cudaError_t launch_lm_head(const RowMap& m, const Model& md, KvState& kv,
-                           float* logits, cudaStream_t st);
 cudaError_t launch_accept(const RowMap& m, const Model& md, KvState& kv,
                           const int32_t* cand, const as2d_verify_out& out,
                           cudaStream_t st);
 cudaError_t launch_rollback(KvState& kv, const int32_t* new_len,
                             const int32_t* new_root, cudaStream_t st);
+// Load-time weight re-layout (k_pack.cu).
+size_t packed_elems(int n_rows, int K);
+cudaError_t pack_weights(bf16* dst, int n_rows, int K, const void* const* segs,
+                         const int* seg_rows, int nseg, bool interleave, cudaStream_t st);
+
+// Split-KV attention on the tensor cores + partition merge (k_attn.cu).
+int attn_partitions(int capacity);
+cudaError_t launch_attention_split(const RowMap& m, const Model& md, KvState& kv, int layer,
+                                   cudaStream_t st);
+
+// Tensor-core GEMM launchers (k_tc_*.cu), one per fused epilogue.
+cudaError_t tc_gemm_qkv(int nb, const CUtensorMap& x, const TcParams& p,
+                        cudaStream_t st);
+cudaError_t tc_gemm_resid(int nb, const CUtensorMap& x, const TcParams& p,
+                          cudaStream_t st);
+cudaError_t tc_gemm_swiglu(int nb, const CUtensorMap& x, const TcParams& p,
+                           cudaStream_t st);
+cudaError_t tc_gemm_logits(int nb, const CUtensorMap& x, const TcParams& p,
+                           cudaStream_t st);
+
 cudaError_t launch_f32_from_bf16(float* dst, const void* src, int64_t n,
                                  cudaStream_t st);
 

@@ -1,0 +1,480 @@
+// gemm_tc.cuh -- skinny GEMM on the 5th-generation tensor cores for the
+// verification pass: D[n][m] = sum_k W[n][k] X[m][k] for the k + 1 token rows
+// m of a block (a handful) and every output feature n of a weight matrix W.
+//
+// Design (weights streamed once per block from HBM):
+//   * swap-AB: the 128-row weight tile is the MMA's M operand (tcgen05.mma
+//     kind::f16, M = 128), the token rows, padded to NB in {16..256}, are its
+//     N operand, so no tensor-core work is spent on padding weight rows;
+//   * weights are stored tile-major at load time (k_pack.cu): every 128 x 64
+//     weight tile is one contiguous, pre-swizzled 16 KB block, fetched with a
+//     single bulk copy (cp.async.bulk), so each SM streams one contiguous
+//     region; the NB x 64 activation tiles come by TMA (cp.async.bulk.tensor,
+//     128-byte swizzle).  An S-deep shared-memory ring guarded by mbarriers;
+//     one thread issues loads, one thread issues MMAs, four warps drain the
+//     fp32 accumulator from TMEM (double-buffered);
+//   * stream-K: the (tile, 64-column k-block) units are split evenly over a
+//     persistent grid of one CTA per SM, so every SM streams the same number
+//     of weight bytes whatever N is.  A tile cut between CTAs is finished by
+//     the last CTA to arrive (an arrival counter, no waiting), which adds the
+//     partial tiles in CTA order: the sum order depends on (N, K, grid) only,
+//     never on the number of token rows, so results are batch invariant;
+//   * the epilogue is fused: RoPE + KV-cache append (QKV), residual add
+//     (O, down), SwiGLU (gate/up), and logits + argmax (LM head).
+// Every mbarrier wait is bounded in time; on expiry the kernel records an
+// error bit, drains its own outstanding copies and MMAs, frees TMEM and exits.
+#pragma once
+
+#include "as2d_internal.h"
+#include "ptx_sm100.cuh"
+
+#ifndef AS2D_RING16
+#define AS2D_RING16 5
+#endif
+
+namespace as2d {
+
+template <int NB>
+struct TcShape {
+  // ring depth: about 160 KB of weight tiles in flight per SM
+  static constexpr int S = NB == 16 ? AS2D_RING16 : NB == 32 ? 5 : NB == 64 ? 5 : NB == 128 ? 4 : 3;
+  static constexpr uint32_t A_BYTES = 128 * 64 * 2;
+  static constexpr uint32_t B_BYTES = NB * 64 * 2;
+  static constexpr int CH = 16;       // epilogue column chunk
+  static constexpr int SP = CH + 1;   // padded shared-memory row
+  static constexpr uint32_t TMEM_COLS = (2 * NB < 32) ? 32 : 2 * NB;
+  static constexpr uint32_t SMEM =
+      1024 + S * (A_BYTES + B_BYTES) + 128 * SP * 4 + (NB + 64) * 4 + (2 * S + 5) * 8 + 16;
+};
+
+__device__ __forceinline__ float tc_silu(float x) { return x / (1.0f + expf(-x)); }
+
+__device__ __forceinline__ unsigned long long tc_pack_best(float v, int idx) {
+  uint32_t u = __float_as_uint(v);
+  uint32_t key = (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+  return ((unsigned long long)key << 32) | (unsigned long long)(0xFFFFFFFFu - (uint32_t)idx);
+}
+
+__device__ __forceinline__ long long tc_start(int c, const TcParams& p) {
+  return (long long)c * p.units / p.grid;
+}
+__device__ __forceinline__ int tc_owner(long long u, const TcParams& p) {
+  return (int)(((u + 1) * (long long)p.grid - 1) / p.units);
+}
+
+// Fused epilogue of one 16-row chunk: sC[n * SP + j] holds D for tile row n
+// and token row row0 + m0 + j.  Runs on the 128 epilogue threads (et).
+template <int NB, int EPI>
+__device__ __forceinline__ void tc_epilogue_chunk(const TcParams& p, const float* sC, float* red,
+                                                  int tile, int m0, int et) {
+  constexpr int SP = TcShape<NB>::SP;
+  constexpr int CH = TcShape<NB>::CH;
+  if (EPI == TC_RESID) {
+    // thread et owns tile row n = et for the chunk's 16 token rows: all
+    // residual loads are issued before any add, so they overlap.  The new
+    // residual also yields the next projection's operand and its share of
+    // the row's sum of squares (warp butterflies, then warps in order).
+    const int n = et, col = tile * 128 + n;
+    const float gn = p.g_next[col];
+    float hv[CH];
+#pragma unroll
+    for (int j = 0; j < CH; ++j)
+      if (m0 + j < p.rows) hv[j] = p.h[(size_t)(p.row0 + m0 + j) * p.N + col];
+#pragma unroll
+    for (int j = 0; j < CH; ++j) {
+      if (m0 + j < p.rows) {
+        const size_t at = (size_t)(p.row0 + m0 + j) * p.N + col;
+        const float hn = hv[j] + sC[n * SP + j];
+        p.h[at] = hn;
+        p.xn[at] = __float2bfloat16_rn(hn * gn);
+        hv[j] = hn * hn;
+      } else {
+        hv[j] = 0.f;
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < CH; ++j) {
+      float v = hv[j];
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
+      if ((et & 31) == 0) red[(et >> 5) * CH + j] = v;
+    }
+    ptx::named_bar_sync(1, 128);
+    if (et < CH && m0 + et < p.rows)
+      p.ss[(size_t)tile * p.ss_ld + p.row0 + m0 + et] =
+          ((red[et] + red[CH + et]) + red[2 * CH + et]) + red[3 * CH + et];
+  } else if (EPI == TC_SWIGLU) {
+    const int F = p.N >> 1;
+    for (int idx = et; idx < 64 * CH; idx += 128) {
+      const int j = idx >> 6, i = idx & 63, m = m0 + j;
+      if (m >= p.rows) break;
+      const float g = sC[i * SP + j], up = sC[(64 + i) * SP + j];
+      p.u[(size_t)(p.row0 + m) * F + (size_t)tile * 64 + i] = __float2bfloat16_rn(tc_silu(g) * up);
+    }
+  } else if (EPI == TC_QKV) {
+    const int d = p.d, half = d >> 1, q_dim = p.nq * d;
+    for (int idx = et; idx < 128 * CH; idx += 128) {
+      const int j = idx >> 7, n = idx & 127, m = m0 + j;
+      if (m >= p.rows) break;
+      const int gm = p.row0 + m;
+      const int col = tile * 128 + n, head = col / d, e = col - head * d;
+      const float x = sC[n * SP + j];
+      if (head < p.nq + p.nkv) {
+        const int i = e < half ? e : e - half;
+        const float2 cs = p.rope[(size_t)gm * half + i];
+        float y;
+        if (e < half) {
+          y = x * cs.x - sC[(n + half) * SP + j] * cs.y;
+        } else {
+          y = x * cs.x + sC[(n - half) * SP + j] * cs.y;
+        }
+        if (head < p.nq) {
+          p.q[(size_t)gm * q_dim + col] = y;
+        } else {
+          const int b = row_request(p.rm, gm);
+          const int pos = p.len[b] + (gm - p.rm.start[b]);
+          const size_t off =
+              ((((size_t)p.layer * p.batch + b) * p.nkv + (head - p.nq)) * p.cap + pos) * d + e;
+          p.kc[off] = __float2bfloat16_rn(y);
+        }
+      } else {
+        const int b = row_request(p.rm, gm);
+        const int pos = p.len[b] + (gm - p.rm.start[b]);
+        const size_t off =
+            ((((size_t)p.layer * p.batch + b) * p.nkv + (head - p.nq - p.nkv)) * p.cap + pos) * d + e;
+        p.vc[off] = __float2bfloat16_rn(x);
+      }
+    }
+  } else {  // TC_LOGITS
+    if (p.logits) {
+      for (int idx = et; idx < 128 * CH; idx += 128) {
+        const int j = idx >> 7, n = idx & 127, m = m0 + j;
+        if (m >= p.rows) break;
+        const int col = tile * 128 + n;
+        if (col < p.N) p.logits[(size_t)(p.row0 + m) * p.N + col] = sC[n * SP + j];
+      }
+    }
+    const int ew = et >> 5, el = et & 31;
+    for (int j = ew; j < CH; j += 4) {
+      const int m = m0 + j;
+      if (m >= p.rows) break;
+      unsigned long long best = 0ull;
+#pragma unroll
+      for (int t = 0; t < 4; ++t) {
+        const int n = el + 32 * t, col = tile * 128 + n;
+        if (col < p.N) {
+          const unsigned long long key = tc_pack_best(sC[n * SP + j], col);
+          best = key > best ? key : best;
+        }
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        const unsigned long long other = __shfl_xor_sync(0xFFFFFFFFu, best, o);
+        best = other > best ? other : best;
+      }
+      if (el == 0) atomicMax(&p.best[p.row0 + m], best);
+    }
+  }
+}
+
+template <int NB, int EPI>
+__global__ void __launch_bounds__(192, 1)
+    tc_gemm_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ TcParams p) {
+  using Sh = TcShape<NB>;
+  constexpr int S = Sh::S;
+  constexpr uint32_t A_BYTES = Sh::A_BYTES, B_BYTES = Sh::B_BYTES;
+  constexpr int CH = Sh::CH, SP = Sh::SP;
+  constexpr uint32_t IDESC = ptx::idesc_bf16_f32(128, NB);
+
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = sA + S * A_BYTES;
+  float* sC = reinterpret_cast<float*>(sB + S * B_BYTES);
+  float* s_rinv = sC + 128 * SP;  // [NB] 1 / rms of each token row (normed inputs)
+  float* red = s_rinv + NB;       // [64] cross-warp reduction scratch
+  uint64_t* full = reinterpret_cast<uint64_t*>(red + 64);
+  uint64_t* empty = full + S;
+  uint64_t* acc_full = empty + S;   // [2]
+  uint64_t* acc_empty = acc_full + 2;  // [2]
+  uint64_t* drain = acc_empty + 2;     // [1]
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  int* flags = reinterpret_cast<int*>(tmem_slot + 2);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int c = blockIdx.x;
+  const long long u0 = tc_start(c, p), u1 = tc_start(c + 1, p);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      ptx::mbar_init(&full[s], 1);
+      ptx::mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      ptx::mbar_init(&acc_full[b], 1);
+      ptx::mbar_init(&acc_empty[b], 4);
+    }
+    ptx::mbar_init(drain, 1);
+    flags[0] = 0;
+    flags[1] = 0;
+    ptx::fence_mbar_init();
+  }
+  if (warp == 1) ptx::tmem_alloc(tmem_slot, Sh::TMEM_COLS);
+  ptx::tc_fence_before();
+  __syncthreads();
+  ptx::tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  ptx::griddep_launch_dependents();
+
+  if (warp == 0) {
+    // ---------------- TMA producer ----------------
+    if (lane == 0) {
+      ptx::prefetch_tmap(&tmX);
+      const uint64_t pol_w = ptx::policy_evict_first();
+      const uint64_t pol_x = ptx::policy_evict_last();
+      // Weight tiles do not depend on earlier kernels: the first ring's worth
+      // is requested before waiting for the predecessor, the activation tiles
+      // after it.
+      const long long npre_ll = (u1 - u0) < S ? (u1 - u0) : S;
+      const int npre = (int)npre_ll;
+      for (int it = 0; it < npre; ++it) {
+        const long long u = u0 + it;
+        ptx::mbar_arrive_expect_tx(&full[it], A_BYTES + B_BYTES);
+        ptx::bulk_load(sA + it * A_BYTES, p.w + (size_t)u * (128 * 64), A_BYTES, &full[it], pol_w);
+      }
+      ptx::griddep_wait();
+      for (int it = 0; it < npre; ++it) {
+        const long long u = u0 + it;
+        const int kb = (int)(u - (u / p.kb) * (long long)p.kb);
+        ptx::tma_load_2d(sB + it * B_BYTES, &tmX, &full[it], kb * 64, p.row0, pol_x);
+      }
+      int it = npre;
+      bool ok = true;
+      for (long long u = u0 + npre; u < u1; ++u, ++it) {
+        const int s = it % S;
+        const uint32_t ph = (uint32_t)(it / S) & 1u;
+        if (!ptx::mbar_wait(&empty[s], ph ^ 1u, p.timeout_ns)) {
+          ok = false;
+          break;
+        }
+        const int kb = (int)(u - (u / p.kb) * (long long)p.kb);
+        ptx::mbar_arrive_expect_tx(&full[s], A_BYTES + B_BYTES);
+        ptx::bulk_load(sA + s * A_BYTES, p.w + (size_t)u * (128 * 64), A_BYTES, &full[s], pol_w);
+        ptx::tma_load_2d(sB + s * B_BYTES, &tmX, &full[s], kb * 64, p.row0, pol_x);
+      }
+      if (!ok) {
+        atomicOr(p.err, kErrTimeout);
+        flags[0] = 1;
+      }
+      // every copy this CTA issued has landed before the CTA may exit
+      for (int j = (it > S ? it - S : 0); j < it; ++j)
+        ptx::mbar_wait(&full[j % S], (uint32_t)(j / S) & 1u, p.timeout_ns);
+    }
+  } else if (warp == 1) {
+    // ---------------- MMA issuer ----------------
+    if (lane == 0) {
+      int it = 0, seg = 0;
+      bool ok = true;
+      for (long long u = u0; u < u1 && ok; ++seg) {
+        const int tile = (int)(u / p.kb);
+        const long long tend = (long long)(tile + 1) * p.kb;
+        const long long send = u1 < tend ? u1 : tend;
+        const int buf = seg & 1;
+        const uint32_t bph = (uint32_t)(seg >> 1) & 1u;
+        if (!ptx::mbar_wait(&acc_empty[buf], bph ^ 1u, p.timeout_ns)) {
+          ok = false;
+          break;
+        }
+        ptx::tc_fence_after();
+        const uint32_t dt = tmem + (uint32_t)(buf * NB);
+        for (long long v = u; v < send; ++v, ++it) {
+          const int s = it % S;
+          const uint32_t ph = (uint32_t)(it / S) & 1u;
+          if (!ptx::mbar_wait(&full[s], ph, p.timeout_ns)) {
+            ok = false;
+            break;
+          }
+          ptx::tc_fence_after();
+          const uint64_t ad = ptx::sdesc_sw128(ptx::smem_u32(sA + s * A_BYTES));
+          const uint64_t bd = ptx::sdesc_sw128(ptx::smem_u32(sB + s * B_BYTES));
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)
+            ptx::mma_bf16(dt, ad + 2 * kk, bd + 2 * kk, IDESC, (v > u || kk > 0) ? 1u : 0u);
+          ptx::mma_commit(&empty[s]);
+        }
+        if (!ok) break;
+        ptx::mma_commit(&acc_full[buf]);
+        u = send;
+      }
+      if (!ok) {
+        atomicOr(p.err, kErrTimeout);
+        flags[0] = 1;
+      }
+      // every MMA this thread issued has completed before TMEM is freed
+      ptx::mma_commit(drain);
+      ptx::mbar_wait(drain, 0, p.timeout_ns);
+    }
+  } else {
+    // ---------------- epilogue: warps 2..5, one TMEM lane each ----------------
+    ptx::griddep_wait();  // the epilogue reads and writes the predecessors' outputs
+    const int q4 = warp & 3;
+    const int nl = q4 * 32 + lane;  // tile row this thread drains
+    const int et = threadIdx.x - 64;
+    if (EPI != TC_RESID) {
+      // 1 / rms of each token row from the producer's per-tile sums (in order)
+      for (int m = et; m < p.rows; m += 128) {
+        const float* src = p.ss + p.row0 + m;
+        float tot = 0.f;
+        for (int t0 = 0; t0 < p.n_htiles; t0 += 8) {
+          float v[8];
+#pragma unroll
+          for (int u = 0; u < 8; ++u)
+            v[u] = (t0 + u < p.n_htiles) ? src[(size_t)(t0 + u) * p.ss_ld] : 0.f;
+#pragma unroll
+          for (int u = 0; u < 8; ++u) tot += v[u];
+        }
+        s_rinv[m] = rsqrtf(tot / (float)p.hidden + p.eps);
+      }
+      ptx::named_bar_sync(1, 128);
+    }
+    const int nchunks = (p.rows + CH - 1) / CH;
+    const int first_tile = (int)(u0 / p.kb);
+    int seg = 0;
+    for (long long u = u0; u < u1; ++seg) {
+      const int tile = (int)(u / p.kb);
+      const long long tstart = (long long)tile * p.kb, tend = tstart + p.kb;
+      const long long send = u1 < tend ? u1 : tend;
+      const bool whole = (u == tstart && send == tend);
+      const int buf = seg & 1;
+      const uint32_t bph = (uint32_t)(seg >> 1) & 1u;
+      if (!ptx::mbar_wait(&acc_full[buf], bph, p.timeout_ns)) {
+        atomicOr(p.err, kErrTimeout);
+        break;
+      }
+      ptx::tc_fence_after();
+      const uint32_t tbase = tmem + (uint32_t)(buf * NB) + ((uint32_t)(q4 * 32) << 16);
+      if (whole) {
+        for (int ch = 0; ch < nchunks; ++ch) {
+          uint32_t v[16];
+          ptx::tmem_ld16(tbase + ch * CH, v);
+          ptx::tmem_ld_wait();
+          ptx::named_bar_sync(1, 128);
+#pragma unroll
+          for (int j = 0; j < CH; ++j)
+            sC[nl * SP + j] = (EPI == TC_RESID) ? __uint_as_float(v[j])
+                                                : __uint_as_float(v[j]) * s_rinv[ch * CH + j];
+          ptx::named_bar_sync(1, 128);
+          tc_epilogue_chunk<NB, EPI>(p, sC, red, tile, ch * CH, et);
+        }
+        ptx::tc_fence_before();
+        __syncwarp();
+        if (lane == 0) ptx::mbar_arrive(&acc_empty[buf]);
+      } else {
+        const int slot = (tile == first_tile) ? 0 : 1;
+        // partial tile, laid out [n][NB]: a thread's token rows are contiguous
+        float* wsp = p.ws + ((size_t)(c * 2 + slot) * 128 + nl) * NB;
+        for (int ch = 0; ch < nchunks; ++ch) {
+          uint32_t v[16];
+          ptx::tmem_ld16(tbase + ch * CH, v);
+          ptx::tmem_ld_wait();
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+            *reinterpret_cast<float4*>(wsp + ch * CH + 4 * q) =
+                make_float4(__uint_as_float(v[4 * q]), __uint_as_float(v[4 * q + 1]),
+                            __uint_as_float(v[4 * q + 2]), __uint_as_float(v[4 * q + 3]));
+        }
+        ptx::tc_fence_before();
+        __syncwarp();
+        if (lane == 0) ptx::mbar_arrive(&acc_empty[buf]);
+        __threadfence();
+        ptx::named_bar_sync(1, 128);
+        const int c_first = tc_owner(tstart, p), c_last = tc_owner(tend - 1, p);
+        const int nparts = c_last - c_first + 1;
+        if (et == 0) flags[1] = (atomicAdd(&p.counters[tile], 1) == nparts - 1) ? 1 : 0;
+        ptx::named_bar_sync(1, 128);
+        if (flags[1]) {
+          __threadfence();
+          for (int ch = 0; ch < nchunks; ++ch) {
+            // partial tiles added in CTA order; each part's 16 loads are
+            // independent, so a part costs one round trip to L2
+            float acc[CH];
+#pragma unroll
+            for (int j = 0; j < CH; ++j) acc[j] = 0.f;
+            const int live = p.rows - ch * CH;  // token rows of this chunk that exist
+            for (int part0 = 0; part0 < nparts; part0 += 4) {
+              float4 v[4][4];
+#pragma unroll
+              for (int pp = 0; pp < 4; ++pp) {
+                if (part0 + pp < nparts) {
+                  const int cp = c_first + part0 + pp;
+                  const int sl = ((int)(tc_start(cp, p) / p.kb) == tile) ? 0 : 1;
+                  const float* src = p.ws + ((size_t)(cp * 2 + sl) * 128 + nl) * NB + ch * CH;
+#pragma unroll
+                  for (int q = 0; q < 4; ++q)
+                    if (4 * q < live) v[pp][q] = __ldcg(reinterpret_cast<const float4*>(src) + q);
+                }
+              }
+#pragma unroll
+              for (int pp = 0; pp < 4; ++pp) {
+                if (part0 + pp < nparts) {
+#pragma unroll
+                  for (int q = 0; q < 4; ++q) {
+                    if (4 * q < live) {
+                      acc[4 * q] += v[pp][q].x;
+                      acc[4 * q + 1] += v[pp][q].y;
+                      acc[4 * q + 2] += v[pp][q].z;
+                      acc[4 * q + 3] += v[pp][q].w;
+                    }
+                  }
+                }
+              }
+            }
+            ptx::named_bar_sync(1, 128);
+#pragma unroll
+            for (int j = 0; j < CH; ++j)
+              sC[nl * SP + j] = (EPI == TC_RESID) ? acc[j] : acc[j] * s_rinv[ch * CH + j];
+            ptx::named_bar_sync(1, 128);
+            tc_epilogue_chunk<NB, EPI>(p, sC, red, tile, ch * CH, et);
+          }
+          if (et == 0) p.counters[tile] = 0;
+        }
+      }
+      u = send;
+    }
+  }
+
+  ptx::tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    ptx::tc_fence_after();
+    ptx::tmem_dealloc(tmem, Sh::TMEM_COLS);
+  }
+}
+
+template <int NB, int EPI>
+cudaError_t tc_gemm_launch(const CUtensorMap& x, const TcParams& p, cudaStream_t st) {
+  constexpr uint32_t smem = TcShape<NB>::SMEM;
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(tc_gemm_kernel<NB, EPI>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  return launch_pdl(tc_gemm_kernel<NB, EPI>, dim3(p.grid), dim3(192), smem, st, x, p);
+}
+
+template <int EPI>
+cudaError_t tc_gemm_dispatch(int nb, const CUtensorMap& x, const TcParams& p, cudaStream_t st) {
+  switch (nb) {
+    case 16: return tc_gemm_launch<16, EPI>(x, p, st);
+    case 32: return tc_gemm_launch<32, EPI>(x, p, st);
+    case 64: return tc_gemm_launch<64, EPI>(x, p, st);
+    case 128: return tc_gemm_launch<128, EPI>(x, p, st);
+    case 256: return tc_gemm_launch<256, EPI>(x, p, st);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace as2d

@@ -53,7 +53,9 @@ class ModelConfig:
 TINY = ModelConfig("tiny", 2, 256, 4, 2, 64, 704, 4096)
 M1P5B = ModelConfig("1.5b", 28, 1536, 12, 2, 128, 8960, 151936)
 M7B = ModelConfig("7b", 28, 3584, 28, 4, 128, 18944, 152064)
-MODELS = {m.name: m for m in (TINY, M1P5B, M7B)}
+# 7B-shaped decoder with two layers: small enough for profiler captures
+M7B_2L = ModelConfig("7b-2l", 2, 3584, 28, 4, 128, 18944, 152064)
+MODELS = {m.name: m for m in (TINY, M1P5B, M7B, M7B_2L)}
 
 # ---- stream ids ------------------------------------------------------------
 S_EMBED, S_LM_HEAD, S_FINAL_NORM = 1, 2, 3

@@ -20,8 +20,8 @@ def declared_entry_points():
 
 @pytest.fixture(scope="module")
 def lib():
-    from paper_2609_37617_gb300 import build
-    build.build()
+    import __graft_entry__
+    __graft_entry__._lib_build_module().build()
     import paper_2609_37617_gb300 as p
     return p
 
