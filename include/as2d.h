@@ -170,6 +170,35 @@ as2d_status as2d_kv_device_state(as2d_kv* kv, const int32_t** len,
    AS2D_OK. */
 as2d_status as2d_kv_check(as2d_kv* kv, void* stream);
 
+/* One greedy decode step (k = 0) of a single request that allocates no
+   memory.  The paper has no counterpart: this is for callers that must not
+   allocate device memory when they decode -- for example a process whose
+   device memory is handed out by another component under a fixed budget, or
+   a real-time loop that cannot accept the latency or the possible failure of
+   an allocation.  The model must have been loaded (as2d_model_load allocates,
+   once, at set-up).  Every other byte a call needs lives in one array of
+   8,866,560 bytes compiled into the library; each GPU that loads the library
+   holds it until the process exits.
+   k_cache, v_cache: device bf16 [n_layers][1][n_kv][capacity][head_dim] as
+   for as2d_kv_init_prefilled.  len, root: device int32 [1], the request's
+   state, updated in place (len += 1, root = correction) as by
+   as2d_decode_step.  correction_token: device int32 [1].  logits: device
+   float [vocab] or NULL.
+   Limits (AS2D_ERR_CAPACITY / AS2D_ERR_UNSUPPORTED on the host, before any
+   work): capacity <= 4096, hidden <= 4096, ffn <= 20480, n_q * head_dim <=
+   4096, n_kv <= 8, n_q / n_kv <= 16, vocab <= 262144, at most 192 SMs.
+   The first call on a device (and the first after a model of another shape)
+   looks up the array's device address and builds descriptors of it; make
+   that first call before any stream capture.  All calls share the one
+   array and each call starts by clearing the parts that must start at zero,
+   so calls that overlap on the GPU (other streams, other host threads) race
+   and give wrong results: issue them one after another.  Device-side
+   errors of this entry point are not reported through as2d_kv_check. */
+as2d_status as2d_decode_step_static(as2d_model* model, void* k_cache, void* v_cache,
+                                    int32_t capacity, int32_t* len, int32_t* root,
+                                    int32_t* correction_token, float* logits,
+                                    void* stream);
+
 /* Measurement support (not part of the verification step).  Kernel classes
    of one verification pass, in launch order per layer: */
 #define AS2D_KERNEL_QKV 0        /* norm + QKV projection               */

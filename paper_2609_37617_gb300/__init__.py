@@ -32,7 +32,7 @@ EXPORTED = ("as2d_model_load", "as2d_kv_init_prefilled", "as2d_verify_block",
             "as2d_decode_step", "as2d_kv_rollback", "as2d_kv_read_state",
             "as2d_kv_device_state", "as2d_kv_check", "as2d_kv_free",
             "as2d_model_free", "as2d_last_error", "as2d_kv_profile",
-            "as2d_kv_profile_read")
+            "as2d_kv_profile_read", "as2d_decode_step_static")
 KERNEL_CLASSES = {"qkv": 0, "attention": 1, "o": 2, "gate_up": 3, "down": 4,
                   "lm_head": 5, "other": 6}
 
@@ -87,6 +87,8 @@ _lib.as2d_kv_profile_read.argtypes = [_P, ctypes.POINTER(ctypes.c_int32),
                                       ctypes.POINTER(ctypes.c_double),
                                       ctypes.POINTER(ctypes.c_int64)]
 _lib.as2d_kv_profile_read.restype = _S
+_lib.as2d_decode_step_static.argtypes = [_P, _P, _P, ctypes.c_int32, _P, _P, _P, _P, _P]
+_lib.as2d_decode_step_static.restype = _S
 _lib.as2d_last_error.argtypes = []
 _lib.as2d_last_error.restype = ctypes.c_char_p
 
@@ -198,6 +200,16 @@ def as2d_kv_profile_read(kv):
     alln = ctypes.c_int64()
     st = _lib.as2d_kv_profile_read(_P(kv), ctypes.byref(n), ctypes.byref(ms), ctypes.byref(alln))
     return st, n.value, ms.value, alln.value
+
+
+def as2d_decode_step_static(model, k_cache_ptr, v_cache_ptr, capacity, len_ptr, root_ptr,
+                            correction_ptr, logits_ptr=0, stream=0):
+    """Single-request decode step whose working memory is the library's fixed
+    array (no allocation); see include/as2d.h."""
+    return _lib.as2d_decode_step_static(_P(model), _P(int(k_cache_ptr)), _P(int(v_cache_ptr)),
+                                        int(capacity), _P(int(len_ptr)), _P(int(root_ptr)),
+                                        _P(int(correction_ptr)), _P(int(logits_ptr) or None),
+                                        _P(int(stream) or None))
 
 
 def exported_symbols():

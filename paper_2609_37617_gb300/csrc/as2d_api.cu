@@ -562,3 +562,192 @@ extern "C" as2d_status as2d_kv_profile_read(as2d_kv* kh, int32_t* launches,
   s.launches = 0;
   return AS2D_OK;
 }
+
+// ---- decode step with no allocation -------------------------------------------
+//
+// For callers that must not allocate device memory when they decode: for
+// example a process whose device memory is handed out by another component
+// under a fixed budget, or a real-time loop where the latency or the possible
+// failure of an allocation is not acceptable.  The model is loaded once
+// beforehand (that allocates, at set-up time); each call then keeps all of its
+// working memory in one array compiled into this library, so it calls no
+// allocator at all.
+
+namespace {
+
+constexpr int kStaticMaxHidden = 4096;
+constexpr int kStaticMaxFfn = 20480;
+constexpr int kStaticMaxQDim = 4096;     // n_q * head_dim
+constexpr int kStaticMaxKvHeads = 8;
+constexpr int kStaticMaxGroup = 16;      // n_q / n_kv
+constexpr int kStaticMaxCapacity = 4096;
+constexpr int kStaticMaxVocab = 262144;
+constexpr int kStaticMaxSms = 192;
+constexpr int kStaticRows = 16;          // one token row, padded to a TMA box
+constexpr int kStaticParts = kStaticMaxCapacity / 64;
+
+constexpr size_t sa(size_t x) { return (x + 255) / 256 * 256; }
+constexpr size_t kOffErr = 0;                                                     // err, bad, n
+constexpr size_t kOffH = kOffErr + 256;
+constexpr size_t kOffXn = kOffH + sa((size_t)kStaticRows * kStaticMaxHidden * 4);
+constexpr size_t kOffQ = kOffXn + sa((size_t)kStaticRows * kStaticMaxHidden * 2);
+constexpr size_t kOffAo = kOffQ + sa((size_t)kStaticRows * kStaticMaxQDim * 4);
+constexpr size_t kOffU = kOffAo + sa((size_t)kStaticRows * kStaticMaxQDim * 2);
+constexpr size_t kOffBest = kOffU + sa((size_t)kStaticRows * kStaticMaxFfn * 2);
+constexpr size_t kOffRope = kOffBest + sa((size_t)kStaticRows * 8);
+constexpr size_t kOffSs = kOffRope + sa((size_t)kStaticRows * 64 * 8);
+constexpr size_t kOffWs = kOffSs + sa((size_t)(kStaticMaxHidden / 128) * kStaticRows * 4);
+constexpr size_t kOffCnt = kOffWs + sa((size_t)kStaticMaxSms * 2 * 16 * 128 * 4);
+constexpr size_t kOffAttnO = kOffCnt + sa((size_t)(kStaticMaxVocab / 128 + 64) * 4);
+constexpr size_t kOffAttnMl =
+    kOffAttnO + sa((size_t)kStaticMaxKvHeads * kStaticParts * kStaticMaxGroup * 128 * 4);
+constexpr size_t kStaticScratchBytes =
+    kOffAttnMl + sa((size_t)kStaticMaxKvHeads * kStaticParts * kStaticMaxGroup * 8);
+
+struct StaticDevice {
+  bool ready = false;
+  char* base = nullptr;
+  CUtensorMap tm_xn, tm_ao, tm_u;
+  int hidden = 0, q_dim = 0, ffn = 0;
+};
+constexpr int kStaticMaxDevices = 64;
+StaticDevice g_static_dev[kStaticMaxDevices];
+
+// Host-side descriptor of the scratch, built when the library is loaded so
+// that no call has to allocate it.
+KvState make_static_state() {
+  KvState s;
+  s.len_upper.assign(1, 0);
+  return s;
+}
+KvState g_static_kv = make_static_state();
+
+}  // namespace
+
+// Working memory of as2d_decode_step_static, shared by every call on a device.
+static __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
+
+extern "C" as2d_status as2d_decode_step_static(as2d_model* mh, void* k_cache, void* v_cache,
+                                               int32_t capacity, int32_t* len, int32_t* root,
+                                               int32_t* correction_token, float* logits,
+                                               void* stream) {
+  g_err.clear();
+  if (!mh || !k_cache || !v_cache || !len || !root || !correction_token)
+    return fail(AS2D_ERR_INVALID_ARG, "model, caches, len, root and correction_token are required");
+  const Model& m = mh->m;
+  const as2d_config& c = m.cfg;
+  if (capacity < 1 || capacity > kStaticMaxCapacity)
+    return fail(AS2D_ERR_CAPACITY, "as2d_decode_step_static supports capacity in [1, 4096]");
+  if (c.hidden > kStaticMaxHidden || c.ffn > kStaticMaxFfn || m.q_dim > kStaticMaxQDim ||
+      c.n_kv_heads > kStaticMaxKvHeads || c.n_q_heads / c.n_kv_heads > kStaticMaxGroup ||
+      c.vocab > kStaticMaxVocab || m.sm_count > kStaticMaxSms)
+    return fail(AS2D_ERR_UNSUPPORTED,
+                "model larger than as2d_decode_step_static's fixed working memory (hidden <= "
+                "4096, ffn <= 20480, n_q*head_dim <= 4096, n_kv <= 8, group <= 16, vocab <= "
+                "262144, <= 192 SMs)");
+  int dev = 0;
+  CUDA_TRY(cudaGetDevice(&dev));
+  if (dev < 0 || dev >= kStaticMaxDevices)
+    return fail(AS2D_ERR_UNSUPPORTED, "device ordinal above 63");
+  StaticDevice& sd = g_static_dev[dev];
+  if (!sd.ready || sd.hidden != c.hidden || sd.q_dim != m.q_dim || sd.ffn != c.ffn) {
+    // Set-up, once per device (and again only if a model of another shape is
+    // used): the array's device address, then TMA descriptors of the operand
+    // buffers inside it.  No allocation is involved.
+    void* base = nullptr;
+    CUDA_TRY(cudaGetSymbolAddress(&base, g_static_scratch));
+    char* b = (char*)base;
+    if (!encode_2d(&sd.tm_xn, b + kOffXn, c.hidden, kStaticRows, 64, 16) ||
+        !encode_2d(&sd.tm_ao, b + kOffAo, m.q_dim, kStaticRows, 64, 16) ||
+        !encode_2d(&sd.tm_u, b + kOffU, c.ffn, kStaticRows, 64, 16))
+      return fail(AS2D_ERR_CUDA, "cuTensorMapEncodeTiled failed for the fixed working memory");
+    sd.base = b;
+    sd.hidden = c.hidden;
+    sd.q_dim = m.q_dim;
+    sd.ffn = c.ffn;
+    sd.ready = true;
+  }
+  cudaStream_t st = (cudaStream_t)stream;
+  char* b = sd.base;
+  KvState& s = g_static_kv;
+  s.model = &mh->m;
+  s.batch = 1;
+  s.capacity = capacity;
+  s.k_cache = (bf16*)k_cache;
+  s.v_cache = (bf16*)v_cache;
+  s.len_upper[0] = capacity - 1;  // attention grid covers the whole cache
+  s.d_len = len;
+  s.d_root = root;
+  s.d_err = (int32_t*)(b + kOffErr);
+  s.max_rows = 1;
+  s.rows_alloc = kStaticRows;
+  s.nb_max = 16;
+  s.h = (float*)(b + kOffH);
+  s.xn = (bf16*)(b + kOffXn);
+  s.q = (float*)(b + kOffQ);
+  s.ao = (bf16*)(b + kOffAo);
+  s.u = (bf16*)(b + kOffU);
+  s.best = (unsigned long long*)(b + kOffBest);
+  s.rope = (float2*)(b + kOffRope);
+  s.ss = (float*)(b + kOffSs);
+  s.ws = (float*)(b + kOffWs);
+  s.counters = (int*)(b + kOffCnt);
+  s.attn_o = (float*)(b + kOffAttnO);
+  s.attn_ml = (float2*)(b + kOffAttnMl);
+  s.attn_parts = (capacity + 63) / 64;
+  s.attn_qmax = ((c.n_q_heads / c.n_kv_heads) + 15) / 16 * 16;
+  s.tm_xn[0] = sd.tm_xn;
+  s.tm_ao[0] = sd.tm_ao;
+  s.tm_u[0] = sd.tm_u;
+  s.prof_class = -1;
+  // the array keeps the previous call's contents: clear the error words, the
+  // argmax slots and the stream-K arrival counters, which must start at zero
+  CUDA_TRY(cudaMemsetAsync(b + kOffErr, 0, 256, st));
+  CUDA_TRY(cudaMemsetAsync(b + kOffBest, 0, kStaticRows * 8, st));
+  CUDA_TRY(cudaMemsetAsync(b + kOffCnt, 0, (size_t)(c.vocab / 128 + 64) * 4, st));
+
+  RowMap rm;
+  rm.batch = 1;
+  rm.rows = 1;
+  rm.start[0] = 0;
+  rm.start[1] = 1;
+  as2d_verify_out out{(int32_t*)(b + kOffErr + 16), correction_token, nullptr, logits};
+  const int H = c.hidden, F = c.ffn;
+  LAUNCH(AS2D_KERNEL_OTHER, launch_embed(rm, m, s, nullptr, st));
+  TcParams tp{};
+  tp.h = s.h;
+  tp.u = s.u;
+  tp.q = s.q;
+  tp.kc = s.k_cache;
+  tp.vc = s.v_cache;
+  tp.rope = s.rope;
+  tp.len = s.d_len;
+  tp.batch = 1;
+  tp.cap = capacity;
+  tp.nq = c.n_q_heads;
+  tp.nkv = c.n_kv_heads;
+  tp.d = c.head_dim;
+  tp.logits = logits;
+  tp.best = s.best;
+  tp.xn = s.xn;
+  tp.ss = s.ss;
+  tp.ss_ld = s.rows_alloc;
+  tp.n_htiles = c.hidden / 128;
+  tp.eps = c.rms_eps;
+  tp.hidden = c.hidden;
+  for (int l = 0; l < c.n_layers; ++l) {
+    tp.layer = l;
+    LAUNCH(AS2D_KERNEL_QKV, tc_project(TC_QKV, m, s, rm, m.w_qkv[l], s.tm_xn, m.qkv_rows, H, tp, st));
+    LAUNCH(AS2D_KERNEL_ATTENTION, launch_attention_split(rm, m, s, l, st));
+    tp.g_next = m.mlp_norm[l];
+    LAUNCH(AS2D_KERNEL_O, tc_project(TC_RESID, m, s, rm, m.w_o[l], s.tm_ao, H, m.q_dim, tp, st));
+    LAUNCH(AS2D_KERNEL_GATE_UP, tc_project(TC_SWIGLU, m, s, rm, m.w_gu[l], s.tm_xn, 2 * F, H, tp, st));
+    tp.g_next = (l + 1 < c.n_layers) ? m.attn_norm[l + 1] : m.final_norm;
+    LAUNCH(AS2D_KERNEL_DOWN, tc_project(TC_RESID, m, s, rm, m.w_down[l], s.tm_u, H, F, tp, st));
+  }
+  LAUNCH(AS2D_KERNEL_LM_HEAD, tc_project(TC_LOGITS, m, s, rm, m.lm_head, s.tm_xn, c.vocab, H, tp, st));
+  LAUNCH(AS2D_KERNEL_OTHER, launch_accept(rm, m, s, nullptr, out, st));
+  return AS2D_OK;
+}
+
+static_assert(kStaticScratchBytes == 8866560, "as2d.h states the fixed working-memory size");
