@@ -260,9 +260,9 @@ extern "C" as2d_status as2d_kv_init_prefilled(as2d_model* mh, int32_t batch,
   const size_t R = s.rows_alloc, H = m.cfg.hidden, F = m.cfg.ffn;
   const size_t max_tiles = ((size_t)(m.cfg.vocab > 2 * F ? m.cfg.vocab : 2 * F) + 127) / 128 + 64;
   size_t bytes = 4096 + 3 * align_up((size_t)(batch + 1) * 4, 256);
-  bytes += align_up(R * H * 4, 256) + align_up(R * H * 2, 256) +
+  bytes += align_up(R * H * 4, 256) + align_up(2 * R * H * 2, 256) +
            align_up(R * m.q_dim * 4, 256) +
-           align_up(R * m.q_dim * 2, 256) + align_up(R * F * 2, 256) + align_up(R * 8, 256) +
+           align_up(2 * R * m.q_dim * 2, 256) + align_up(2 * R * F * 2, 256) + align_up(R * 8, 256) +
            align_up(R * (m.cfg.head_dim / 2) * 8, 256) + align_up(R * (H / 128) * 4, 256) +
            align_up((size_t)m.sm_count * 2 * s.nb_max * 128 * 4, 256) + align_up(max_tiles * 4, 256);
   const int group = m.cfg.n_q_heads / m.cfg.n_kv_heads;
@@ -281,10 +281,10 @@ extern "C" as2d_status as2d_kv_init_prefilled(as2d_model* mh, int32_t batch,
   s.d_root = cv.take<int32_t>(batch);
   s.d_err = cv.take<int32_t>(batch + 1);
   s.h = cv.take<float>(R * H);
-  s.xn = cv.take<bf16>(R * H);
+  s.xn = cv.take<bf16>(2 * R * H);
   s.q = cv.take<float>(R * m.q_dim);
-  s.ao = cv.take<bf16>(R * m.q_dim);
-  s.u = cv.take<bf16>(R * F);
+  s.ao = cv.take<bf16>(2 * R * m.q_dim);
+  s.u = cv.take<bf16>(2 * R * F);
   s.best = cv.take<unsigned long long>(R);
   s.rope = cv.take<float2>(R * (m.cfg.head_dim / 2));
   s.ss = cv.take<float>(R * (H / 128));
@@ -296,9 +296,9 @@ extern "C" as2d_status as2d_kv_init_prefilled(as2d_model* mh, int32_t batch,
   for (int i = 0; i < kNbCount && ok; ++i) {
     const int nb = 16 << i;
     if (nb > s.nb_max) break;
-    ok = encode_2d(&s.tm_xn[i], s.xn, H, R, 64, nb) &&
-         encode_2d(&s.tm_ao[i], s.ao, m.q_dim, R, 64, nb) &&
-         encode_2d(&s.tm_u[i], s.u, F, R, 64, nb);
+    ok = encode_2d(&s.tm_xn[i], s.xn, H, 2 * R, 64, nb) &&
+         encode_2d(&s.tm_ao[i], s.ao, m.q_dim, 2 * R, 64, nb) &&
+         encode_2d(&s.tm_u[i], s.u, F, 2 * R, 64, nb);
   }
   if (!ok) {
     cudaFree(s.work);
@@ -434,6 +434,7 @@ as2d_status run_block(KvState& s, const int32_t* cand, const int32_t* k,
   tp.xn = s.xn;
   tp.ss = s.ss;
   tp.ss_ld = s.rows_alloc;
+  tp.lo_row = s.rows_alloc;
   tp.n_htiles = c.hidden / 128;
   tp.eps = c.rms_eps;
   tp.hidden = c.hidden;
@@ -590,10 +591,10 @@ constexpr size_t sa(size_t x) { return (x + 255) / 256 * 256; }
 constexpr size_t kOffErr = 0;                                                     // err, bad, n
 constexpr size_t kOffH = kOffErr + 256;
 constexpr size_t kOffXn = kOffH + sa((size_t)kStaticRows * kStaticMaxHidden * 4);
-constexpr size_t kOffQ = kOffXn + sa((size_t)kStaticRows * kStaticMaxHidden * 2);
+constexpr size_t kOffQ = kOffXn + sa((size_t)2 * kStaticRows * kStaticMaxHidden * 2);
 constexpr size_t kOffAo = kOffQ + sa((size_t)kStaticRows * kStaticMaxQDim * 4);
-constexpr size_t kOffU = kOffAo + sa((size_t)kStaticRows * kStaticMaxQDim * 2);
-constexpr size_t kOffBest = kOffU + sa((size_t)kStaticRows * kStaticMaxFfn * 2);
+constexpr size_t kOffU = kOffAo + sa((size_t)2 * kStaticRows * kStaticMaxQDim * 2);
+constexpr size_t kOffBest = kOffU + sa((size_t)2 * kStaticRows * kStaticMaxFfn * 2);
 constexpr size_t kOffRope = kOffBest + sa((size_t)kStaticRows * 8);
 constexpr size_t kOffSs = kOffRope + sa((size_t)kStaticRows * 64 * 8);
 constexpr size_t kOffWs = kOffSs + sa((size_t)(kStaticMaxHidden / 128) * kStaticRows * 4);
@@ -657,9 +658,9 @@ extern "C" as2d_status as2d_decode_step_static(as2d_model* mh, void* k_cache, vo
     void* base = nullptr;
     CUDA_TRY(cudaGetSymbolAddress(&base, g_static_scratch));
     char* b = (char*)base;
-    if (!encode_2d(&sd.tm_xn, b + kOffXn, c.hidden, kStaticRows, 64, 16) ||
-        !encode_2d(&sd.tm_ao, b + kOffAo, m.q_dim, kStaticRows, 64, 16) ||
-        !encode_2d(&sd.tm_u, b + kOffU, c.ffn, kStaticRows, 64, 16))
+    if (!encode_2d(&sd.tm_xn, b + kOffXn, c.hidden, 2 * kStaticRows, 64, 16) ||
+        !encode_2d(&sd.tm_ao, b + kOffAo, m.q_dim, 2 * kStaticRows, 64, 16) ||
+        !encode_2d(&sd.tm_u, b + kOffU, c.ffn, 2 * kStaticRows, 64, 16))
       return fail(AS2D_ERR_CUDA, "cuTensorMapEncodeTiled failed for the fixed working memory");
     sd.base = b;
     sd.hidden = c.hidden;
@@ -732,6 +733,7 @@ extern "C" as2d_status as2d_decode_step_static(as2d_model* mh, void* k_cache, vo
   tp.xn = s.xn;
   tp.ss = s.ss;
   tp.ss_ld = s.rows_alloc;
+  tp.lo_row = s.rows_alloc;
   tp.n_htiles = c.hidden / 128;
   tp.eps = c.rms_eps;
   tp.hidden = c.hidden;
@@ -750,4 +752,4 @@ extern "C" as2d_status as2d_decode_step_static(as2d_model* mh, void* k_cache, vo
   return AS2D_OK;
 }
 
-static_assert(kStaticScratchBytes == 8866560, "as2d.h states the fixed working-memory size");
+static_assert(kStaticScratchBytes == 9784064, "as2d.h states the fixed working-memory size");

@@ -46,6 +46,7 @@ enum TcEpi { TC_QKV = 0, TC_RESID = 1, TC_SWIGLU = 2, TC_LOGITS = 3 };
 
 struct TcParams {
   const bf16* w;         // packed weight blocks (k_pack.cu), unit u at u * 8192
+  int lo_row;            // operand buffers hold hi rows [0, R), lo rows [R, 2R): R
   int N, K;              // logical W is [N][K]
   int n_tiles, kb;       // 128-row tiles, 64-column k-blocks
   long long units;       // n_tiles * kb
@@ -143,10 +144,11 @@ struct KvState {
   void* work = nullptr;
   size_t work_bytes = 0;
   float* h = nullptr;        // [rows][H] residual stream, fp32
-  bf16* xn = nullptr;        // [rows][H] normalised activations
+  // bf16 operand buffers hold hi rows [0, rows_alloc) then lo rows
+  bf16* xn = nullptr;        // [2 rows][H] next projection's operand bf16(h * g)
   float* q = nullptr;        // [rows][nq][d] rotated queries
-  bf16* ao = nullptr;        // [rows][nq d] attention output
-  bf16* u = nullptr;         // [rows][F] SwiGLU output
+  bf16* ao = nullptr;        // [2 rows][nq d] attention output
+  bf16* u = nullptr;         // [2 rows][F] SwiGLU output
   unsigned long long* best = nullptr;  // [rows] packed (logit, index) maxima
   float2* rope = nullptr;    // [rows][d/2] (cos, sin) at each row's position
   int rows_alloc = 0;        // activation rows allocated (>= every NB used)

@@ -6,6 +6,12 @@
 //   * swap-AB: the 128-row weight tile is the MMA's M operand (tcgen05.mma
 //     kind::f16, M = 128), the token rows, padded to NB in {16..256}, are its
 //     N operand, so no tensor-core work is spent on padding weight rows;
+//   * activations are kept as two bf16 parts, hi = bf16(x) and lo =
+//     bf16(x - hi), stored as two row blocks of the operand buffer; each
+//     k-step issues one MMA per part into the same fp32 accumulator, so the
+//     bf16 weights multiply x to about 16 significant bits (single bf16
+//     operands cost ~5e-2 in the logits of a 28-layer model) at no extra
+//     weight traffic;
 //   * weights are stored tile-major at load time (k_pack.cu): every 128 x 64
 //     weight tile is one contiguous, pre-swizzled 16 KB block, fetched with a
 //     single bulk copy (cp.async.bulk), so each SM streams one contiguous
@@ -29,7 +35,7 @@
 #include "ptx_sm100.cuh"
 
 #ifndef AS2D_RING16
-#define AS2D_RING16 5
+#define AS2D_RING16 6
 #endif
 
 namespace as2d {
@@ -37,14 +43,24 @@ namespace as2d {
 template <int NB>
 struct TcShape {
   // ring depth: about 160 KB of weight tiles in flight per SM
-  static constexpr int S = NB == 16 ? AS2D_RING16 : NB == 32 ? 5 : NB == 64 ? 5 : NB == 128 ? 4 : 3;
+  static constexpr int S = NB == 16 ? AS2D_RING16 : NB == 32 ? 6 : NB == 64 ? 5 : NB == 128 ? 3 : 2;
   static constexpr uint32_t A_BYTES = 128 * 64 * 2;
-  static constexpr uint32_t B_BYTES = NB * 64 * 2;
+  static constexpr uint32_t B_BYTES = NB * 64 * 2;   // one of the hi / lo operand tiles
+  static constexpr uint32_t STAGE_B = 2 * B_BYTES;   // hi tile, then lo tile
   static constexpr int CH = 16;       // epilogue column chunk
   static constexpr int SP = CH + 1;   // padded shared-memory row
-  static constexpr uint32_t TMEM_COLS = (2 * NB < 32) ? 32 : 2 * NB;
+  // hi and lo results accumulate in separate TMEM columns, [0, NB) and
+  // [NB, 2 NB), and are added in the epilogue (hi + lo) -- the same
+  // arithmetic for every NB, so results stay batch invariant.  NB <= 128: one
+  // MMA of N = 2 NB covers the hi and lo rows (adjacent in shared memory) and
+  // reads the weight tile once; NB = 256: two MMAs of N = 256.  Accumulators
+  // are double-buffered while 2 x 2 NB columns fit in TMEM's 512.
+  static constexpr bool ONE_MMA = NB <= 128;
+  static constexpr int ACC_COLS = 2 * NB;
+  static constexpr int NBUF = 2 * ACC_COLS <= 512 ? 2 : 1;
+  static constexpr uint32_t TMEM_COLS = (NBUF * ACC_COLS < 32) ? 32 : NBUF * ACC_COLS;
   static constexpr uint32_t SMEM =
-      1024 + S * (A_BYTES + B_BYTES) + 128 * SP * 4 + (NB + 64) * 4 + (2 * S + 5) * 8 + 16;
+      1024 + S * (A_BYTES + STAGE_B) + 128 * SP * 4 + (NB + 64) * 4 + (2 * S + 5) * 8 + 16;
 };
 
 __device__ __forceinline__ float tc_silu(float x) { return x / (1.0f + expf(-x)); }
@@ -86,7 +102,10 @@ __device__ __forceinline__ void tc_epilogue_chunk(const TcParams& p, const float
         const size_t at = (size_t)(p.row0 + m0 + j) * p.N + col;
         const float hn = hv[j] + sC[n * SP + j];
         p.h[at] = hn;
-        p.xn[at] = __float2bfloat16_rn(hn * gn);
+        const float xv = hn * gn;
+        const bf16 xh = __float2bfloat16_rn(xv);
+        p.xn[at] = xh;
+        p.xn[at + (size_t)p.lo_row * p.N] = __float2bfloat16_rn(xv - __bfloat162float(xh));
         hv[j] = hn * hn;
       } else {
         hv[j] = 0.f;
@@ -109,7 +128,11 @@ __device__ __forceinline__ void tc_epilogue_chunk(const TcParams& p, const float
       const int j = idx >> 6, i = idx & 63, m = m0 + j;
       if (m >= p.rows) break;
       const float g = sC[i * SP + j], up = sC[(64 + i) * SP + j];
-      p.u[(size_t)(p.row0 + m) * F + (size_t)tile * 64 + i] = __float2bfloat16_rn(tc_silu(g) * up);
+      const float uv = tc_silu(g) * up;
+      const bf16 uh = __float2bfloat16_rn(uv);
+      const size_t at = (size_t)(p.row0 + m) * F + (size_t)tile * 64 + i;
+      p.u[at] = uh;
+      p.u[at + (size_t)p.lo_row * F] = __float2bfloat16_rn(uv - __bfloat162float(uh));
     }
   } else if (EPI == TC_QKV) {
     const int d = p.d, half = d >> 1, q_dim = p.nq * d;
@@ -177,21 +200,36 @@ __device__ __forceinline__ void tc_epilogue_chunk(const TcParams& p, const float
   }
 }
 
+// 16 accumulator columns of chunk ch for this thread's TMEM lane: the hi and
+// lo results are added here (hi + lo, fixed order).
+template <int NB>
+__device__ __forceinline__ void tc_load_acc(uint32_t tbase, int ch, uint32_t (&v)[16]) {
+  uint32_t w[16];
+  ptx::tmem_ld16(tbase + ch * 16, v);
+  ptx::tmem_ld16(tbase + NB + ch * 16, w);
+  ptx::tmem_ld_wait();
+#pragma unroll
+  for (int j = 0; j < 16; ++j) v[j] = __float_as_uint(__uint_as_float(v[j]) + __uint_as_float(w[j]));
+}
+
 template <int NB, int EPI>
 __global__ void __launch_bounds__(192, 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ TcParams p) {
   using Sh = TcShape<NB>;
   constexpr int S = Sh::S;
-  constexpr uint32_t A_BYTES = Sh::A_BYTES, B_BYTES = Sh::B_BYTES;
+  constexpr uint32_t A_BYTES = Sh::A_BYTES, B_BYTES = Sh::B_BYTES, STAGE_B = Sh::STAGE_B;
   constexpr int CH = Sh::CH, SP = Sh::SP;
-  constexpr uint32_t IDESC = ptx::idesc_bf16_f32(128, NB);
+  constexpr bool ONE_MMA = Sh::ONE_MMA;
+  constexpr int ACC_COLS = Sh::ACC_COLS;
+  constexpr int NBUF = Sh::NBUF;
+  constexpr uint32_t IDESC = ptx::idesc_bf16_f32(128, ONE_MMA ? 2 * NB : NB);
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   uint8_t* sA = smem;
   uint8_t* sB = sA + S * A_BYTES;
-  float* sC = reinterpret_cast<float*>(sB + S * B_BYTES);
+  float* sC = reinterpret_cast<float*>(sB + S * STAGE_B);
   float* s_rinv = sC + 128 * SP;  // [NB] 1 / rms of each token row (normed inputs)
   float* red = s_rinv + NB;       // [64] cross-warp reduction scratch
   uint64_t* full = reinterpret_cast<uint64_t*>(red + 64);
@@ -240,14 +278,16 @@ __global__ void __launch_bounds__(192, 1)
       const int npre = (int)npre_ll;
       for (int it = 0; it < npre; ++it) {
         const long long u = u0 + it;
-        ptx::mbar_arrive_expect_tx(&full[it], A_BYTES + B_BYTES);
+        ptx::mbar_arrive_expect_tx(&full[it], A_BYTES + STAGE_B);
         ptx::bulk_load(sA + it * A_BYTES, p.w + (size_t)u * (128 * 64), A_BYTES, &full[it], pol_w);
       }
       ptx::griddep_wait();
       for (int it = 0; it < npre; ++it) {
         const long long u = u0 + it;
         const int kb = (int)(u - (u / p.kb) * (long long)p.kb);
-        ptx::tma_load_2d(sB + it * B_BYTES, &tmX, &full[it], kb * 64, p.row0, pol_x);
+        ptx::tma_load_2d(sB + it * STAGE_B, &tmX, &full[it], kb * 64, p.row0, pol_x);
+        ptx::tma_load_2d(sB + it * STAGE_B + B_BYTES, &tmX, &full[it], kb * 64,
+                         p.lo_row + p.row0, pol_x);
       }
       int it = npre;
       bool ok = true;
@@ -259,9 +299,11 @@ __global__ void __launch_bounds__(192, 1)
           break;
         }
         const int kb = (int)(u - (u / p.kb) * (long long)p.kb);
-        ptx::mbar_arrive_expect_tx(&full[s], A_BYTES + B_BYTES);
+        ptx::mbar_arrive_expect_tx(&full[s], A_BYTES + STAGE_B);
         ptx::bulk_load(sA + s * A_BYTES, p.w + (size_t)u * (128 * 64), A_BYTES, &full[s], pol_w);
-        ptx::tma_load_2d(sB + s * B_BYTES, &tmX, &full[s], kb * 64, p.row0, pol_x);
+        ptx::tma_load_2d(sB + s * STAGE_B, &tmX, &full[s], kb * 64, p.row0, pol_x);
+        ptx::tma_load_2d(sB + s * STAGE_B + B_BYTES, &tmX, &full[s], kb * 64, p.lo_row + p.row0,
+                         pol_x);
       }
       if (!ok) {
         atomicOr(p.err, kErrTimeout);
@@ -280,14 +322,14 @@ __global__ void __launch_bounds__(192, 1)
         const int tile = (int)(u / p.kb);
         const long long tend = (long long)(tile + 1) * p.kb;
         const long long send = u1 < tend ? u1 : tend;
-        const int buf = seg & 1;
-        const uint32_t bph = (uint32_t)(seg >> 1) & 1u;
+        const int buf = seg % NBUF;
+        const uint32_t bph = (uint32_t)(seg / NBUF) & 1u;
         if (!ptx::mbar_wait(&acc_empty[buf], bph ^ 1u, p.timeout_ns)) {
           ok = false;
           break;
         }
         ptx::tc_fence_after();
-        const uint32_t dt = tmem + (uint32_t)(buf * NB);
+        const uint32_t dt = tmem + (uint32_t)(buf * ACC_COLS);
         for (long long v = u; v < send; ++v, ++it) {
           const int s = it % S;
           const uint32_t ph = (uint32_t)(it / S) & 1u;
@@ -297,10 +339,20 @@ __global__ void __launch_bounds__(192, 1)
           }
           ptx::tc_fence_after();
           const uint64_t ad = ptx::sdesc_sw128(ptx::smem_u32(sA + s * A_BYTES));
-          const uint64_t bd = ptx::sdesc_sw128(ptx::smem_u32(sB + s * B_BYTES));
+          const uint64_t bh = ptx::sdesc_sw128(ptx::smem_u32(sB + s * STAGE_B));
+          const uint64_t bl = ptx::sdesc_sw128(ptx::smem_u32(sB + s * STAGE_B + B_BYTES));
+          // the operand is x = hi + lo (two bf16 parts), so the weights see x
+          // to about 16 significant bits
 #pragma unroll
-          for (int kk = 0; kk < 4; ++kk)
-            ptx::mma_bf16(dt, ad + 2 * kk, bd + 2 * kk, IDESC, (v > u || kk > 0) ? 1u : 0u);
+          for (int kk = 0; kk < 4; ++kk) {
+            const uint32_t acc = (v > u || kk > 0) ? 1u : 0u;
+            if (ONE_MMA) {
+              ptx::mma_bf16(dt, ad + 2 * kk, bh + 2 * kk, IDESC, acc);
+            } else {
+              ptx::mma_bf16(dt, ad + 2 * kk, bh + 2 * kk, IDESC, acc);
+              ptx::mma_bf16(dt + NB, ad + 2 * kk, bl + 2 * kk, IDESC, acc);
+            }
+          }
           ptx::mma_commit(&empty[s]);
         }
         if (!ok) break;
@@ -346,19 +398,18 @@ __global__ void __launch_bounds__(192, 1)
       const long long tstart = (long long)tile * p.kb, tend = tstart + p.kb;
       const long long send = u1 < tend ? u1 : tend;
       const bool whole = (u == tstart && send == tend);
-      const int buf = seg & 1;
-      const uint32_t bph = (uint32_t)(seg >> 1) & 1u;
+      const int buf = seg % NBUF;
+      const uint32_t bph = (uint32_t)(seg / NBUF) & 1u;
       if (!ptx::mbar_wait(&acc_full[buf], bph, p.timeout_ns)) {
         atomicOr(p.err, kErrTimeout);
         break;
       }
       ptx::tc_fence_after();
-      const uint32_t tbase = tmem + (uint32_t)(buf * NB) + ((uint32_t)(q4 * 32) << 16);
+      const uint32_t tbase = tmem + (uint32_t)(buf * ACC_COLS) + ((uint32_t)(q4 * 32) << 16);
       if (whole) {
         for (int ch = 0; ch < nchunks; ++ch) {
           uint32_t v[16];
-          ptx::tmem_ld16(tbase + ch * CH, v);
-          ptx::tmem_ld_wait();
+          tc_load_acc<NB>(tbase, ch, v);
           ptx::named_bar_sync(1, 128);
 #pragma unroll
           for (int j = 0; j < CH; ++j)
@@ -376,8 +427,7 @@ __global__ void __launch_bounds__(192, 1)
         float* wsp = p.ws + ((size_t)(c * 2 + slot) * 128 + nl) * NB;
         for (int ch = 0; ch < nchunks; ++ch) {
           uint32_t v[16];
-          ptx::tmem_ld16(tbase + ch * CH, v);
-          ptx::tmem_ld_wait();
+          tc_load_acc<NB>(tbase, ch, v);
 #pragma unroll
           for (int q = 0; q < 4; ++q)
             *reinterpret_cast<float4*>(wsp + ch * CH + 4 * q) =

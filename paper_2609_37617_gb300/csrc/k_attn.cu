@@ -11,7 +11,9 @@
 // Pass 1 (attn_part_kernel): one CTA per (64-key partition, kv head, request).
 // Keys and values are staged in shared memory; each warp takes 16 query rows;
 // S = Q K^T and O = P V run on the tensor cores (mma.sync m16n8k16, bf16 in,
-// fp32 accumulate); the softmax runs in fp32 in base 2.  Partition boundaries
+// fp32 accumulate), with Q and P each split into bf16 hi + lo parts (two MMAs)
+// so that only the bf16 cache itself limits precision; the softmax runs in
+// fp32 in base 2.  Partition boundaries
 // are fixed multiples of 64 positions, so a query's partial results do not
 // depend on the other rows of the call (batch invariance).
 // Pass 2 (attn_merge_kernel): per (row, query head) the partitions' (max,
@@ -25,9 +27,13 @@ namespace {
 constexpr int kPart = 64;      // keys per partition (fixed)
 constexpr int kPitch = 136;    // bf16 per shared row: 128 + 8 (272 B, conflict-free)
 
-__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
-  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
-  return *reinterpret_cast<uint32_t*>(&v);
+// x, y -> packed bf16 hi parts and packed bf16 lo parts (x - hi).
+__device__ __forceinline__ void split_bf16x2(float x, float y, uint32_t& hi, uint32_t& lo) {
+  const __nv_bfloat162 h = __floats2bfloat162_rn(x, y);
+  const float2 hf = __bfloat1622float2(h);
+  const __nv_bfloat162 l = __floats2bfloat162_rn(x - hf.x, y - hf.y);
+  hi = *reinterpret_cast<const uint32_t*>(&h);
+  lo = *reinterpret_cast<const uint32_t*>(&l);
 }
 
 __device__ __forceinline__ void mma_16816(float (&c)[4], const uint32_t (&a)[4], uint32_t b0,
@@ -62,7 +68,8 @@ struct AttnArgs {
   float* ws_o;          // [batch][nkv][parts_max][qmax][D]
   float2* ws_ml;        // [batch][nkv][parts_max][qmax] (max, sum), base 2
   int parts_max, qmax;
-  bf16* ao;             // [rows][nq * D]
+  bf16* ao;             // [2 rows][nq * D]: hi rows, then lo rows from lo_row
+  int lo_row;
 };
 
 template <int D>
@@ -122,16 +129,18 @@ __global__ void __launch_bounds__(256, 1) attn_part_kernel(AttnArgs a) {
       float2 xa1 = va ? *reinterpret_cast<const float2*>(qpa + c0 + 8) : make_float2(0.f, 0.f);
       float2 xb0 = vb ? *reinterpret_cast<const float2*>(qpb + c0) : make_float2(0.f, 0.f);
       float2 xb1 = vb ? *reinterpret_cast<const float2*>(qpb + c0 + 8) : make_float2(0.f, 0.f);
-      uint32_t af[4];
-      af[0] = pack_bf16x2(xa0.x * a.qscale, xa0.y * a.qscale);
-      af[1] = pack_bf16x2(xb0.x * a.qscale, xb0.y * a.qscale);
-      af[2] = pack_bf16x2(xa1.x * a.qscale, xa1.y * a.qscale);
-      af[3] = pack_bf16x2(xb1.x * a.qscale, xb1.y * a.qscale);
+      // q as bf16 hi + lo parts: S = Q_hi K^T + Q_lo K^T
+      uint32_t ah[4], al[4];
+      split_bf16x2(xa0.x * a.qscale, xa0.y * a.qscale, ah[0], al[0]);
+      split_bf16x2(xb0.x * a.qscale, xb0.y * a.qscale, ah[1], al[1]);
+      split_bf16x2(xa1.x * a.qscale, xa1.y * a.qscale, ah[2], al[2]);
+      split_bf16x2(xb1.x * a.qscale, xb1.y * a.qscale, ah[3], al[3]);
 #pragma unroll
       for (int nt = 0; nt < 8; ++nt) {
         const uint32_t b0 = *reinterpret_cast<const uint32_t*>(&sK[nt * 8 + gq][c0]);
         const uint32_t b1 = *reinterpret_cast<const uint32_t*>(&sK[nt * 8 + gq][c0 + 8]);
-        mma_16816(s[nt], af, b0, b1);
+        mma_16816(s[nt], ah, b0, b1);
+        mma_16816(s[nt], al, b0, b1);
       }
     }
     // causal mask: row i sees keys up to L + i
@@ -168,13 +177,14 @@ __global__ void __launch_bounds__(256, 1) attn_part_kernel(AttnArgs a) {
     lb += __shfl_xor_sync(0xFFFFFFFFu, lb, 2);
 
     // O = P V: P from the S accumulators (16 x 64), V (64 x D) via ldmatrix.trans
-    uint32_t pf[4][4];
+    // P as bf16 hi + lo parts: O = P_hi V + P_lo V
+    uint32_t pf[4][4], pl[4][4];
 #pragma unroll
     for (int kk = 0; kk < 4; ++kk) {
-      pf[kk][0] = pack_bf16x2(s[2 * kk][0], s[2 * kk][1]);
-      pf[kk][1] = pack_bf16x2(s[2 * kk][2], s[2 * kk][3]);
-      pf[kk][2] = pack_bf16x2(s[2 * kk + 1][0], s[2 * kk + 1][1]);
-      pf[kk][3] = pack_bf16x2(s[2 * kk + 1][2], s[2 * kk + 1][3]);
+      split_bf16x2(s[2 * kk][0], s[2 * kk][1], pf[kk][0], pl[kk][0]);
+      split_bf16x2(s[2 * kk][2], s[2 * kk][3], pf[kk][1], pl[kk][1]);
+      split_bf16x2(s[2 * kk + 1][0], s[2 * kk + 1][1], pf[kk][2], pl[kk][2]);
+      split_bf16x2(s[2 * kk + 1][2], s[2 * kk + 1][3], pf[kk][3], pl[kk][3]);
     }
     const int lr = lane & 7, lm = lane >> 3;
 #pragma unroll
@@ -185,7 +195,9 @@ __global__ void __launch_bounds__(256, 1) attn_part_kernel(AttnArgs a) {
         uint32_t vb4[4];
         ldmatrix_x4_trans(vb4, &sV[kk * 16 + lr + (lm & 1) * 8][dp * 16 + (lm >> 1) * 8]);
         mma_16816(o0, pf[kk], vb4[0], vb4[1]);
+        mma_16816(o0, pl[kk], vb4[0], vb4[1]);
         mma_16816(o1, pf[kk], vb4[2], vb4[3]);
+        mma_16816(o1, pl[kk], vb4[2], vb4[3]);
       }
       const int col = dp * 16 + 2 * tq;
       if (va) {
@@ -261,7 +273,11 @@ __global__ void __launch_bounds__(D) attn_merge_kernel(AttnArgs a) {
     for (int u = 0; u < 32; ++u)
       if (p0 + u < nparts) o += ov[u] * w[p0 + u];
   }
-  a.ao[(size_t)r * a.nq * D + (size_t)j * D + e] = __float2bfloat16_rn(o / s_l);
+  const float ov_ = o / s_l;
+  const bf16 oh = __float2bfloat16_rn(ov_);
+  a.ao[(size_t)r * a.nq * D + (size_t)j * D + e] = oh;
+  a.ao[(size_t)(a.lo_row + r) * a.nq * D + (size_t)j * D + e] =
+      __float2bfloat16_rn(ov_ - __bfloat162float(oh));
 }
 
 }  // namespace
@@ -288,6 +304,7 @@ cudaError_t launch_attention_split(const RowMap& m, const Model& md, KvState& kv
   a.parts_max = kv.attn_parts;
   a.qmax = kv.attn_qmax;
   a.ao = kv.ao;
+  a.lo_row = kv.rows_alloc;
   int64_t max_len = 0;
   for (int b = 0; b < kv.batch; ++b) {
     const int64_t e = kv.len_upper[b] + (m.start[b + 1] - m.start[b]);

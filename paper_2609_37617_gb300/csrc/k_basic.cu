@@ -50,13 +50,17 @@ __global__ void __launch_bounds__(256) embed_kernel(
     tok = 0;
   }
   // residual stream = embedding row; the first projection's operand is
-  // bf16(h * g) and its row sum of squares goes to tile slot 0 (slots 1.. = 0)
+  // h * g as bf16 hi + lo parts (lo rows start at ss_ld = rows allocated) and
+  // its row sum of squares goes to tile slot 0 (slots 1.. = 0)
   const bf16* e = E + (size_t)tok * H;
   float sq = 0.f;
   for (int c = threadIdx.x; c < H; c += blockDim.x) {
     const float x = __bfloat162float(e[c]);
     h[(size_t)r * H + c] = x;
-    xn[(size_t)r * H + c] = __float2bfloat16_rn(x * g0[c]);
+    const float xv = x * g0[c];
+    const bf16 xh = __float2bfloat16_rn(xv);
+    xn[(size_t)r * H + c] = xh;
+    xn[(size_t)(ss_ld + r) * H + c] = __float2bfloat16_rn(xv - __bfloat162float(xh));
     sq = fmaf(x, x, sq);
   }
   sq = warp_sum(sq);

@@ -78,3 +78,21 @@ def compare_block(oracle_res, gpu_logits, gpu_greedy, gpu_n, gpu_corr, k):
     if np.all(sure[: n + 1]):
         assert gpu_n == n and gpu_corr == oracle_res["correction"]
     return d
+
+
+def oracle_block(pair, cache, length, root, cand):
+    """Oracle verification of one block on `cache` (modified in place)."""
+    return pair.oracle.verify_block(cache, length, root, list(cand))
+
+
+def check_parity(ores, gpu, row0, k, where=""):
+    """Compare one request's oracle result with its rows of a GPU call
+    (gpu = (n, corr, greedy, logits) arrays; request at row offset row0)."""
+    n, corr, greedy, logits = gpu
+    d = np.max(np.abs(ores["logits"] - logits[row0:row0 + k + 1]))
+    assert d <= LOGIT_TOL, f"{where}: max |dlogit| = {d}"
+    sure = ores["margin"] > MARGIN_SURE
+    g = greedy[row0:row0 + k + 1]
+    assert np.array_equal(ores["greedy"][sure], g[sure]), where
+    m = ores["n_accepted"]
+    return d, bool(np.all(sure[: m + 1])), m, ores["correction"]
