@@ -33,6 +33,10 @@ METRIC = "7B verify-step µs & committed tok/s vs block k; fraction of HBM roofl
 UNIT = "committed tok/s"
 WORKLOAD = "7b"
 
+# dram__bytes_read.sum + dram__bytes_write.sum per launch from one ncu capture
+# of the kernel as it stands (profiles/); None once the kernel has changed.
+TRAFFIC = {"gate_up": 276091648}  # profiles/gemm_gateup_7b_k8.md
+
 
 def parse():
     ap = argparse.ArgumentParser()
@@ -47,6 +51,9 @@ def parse():
     ap.add_argument("--profile-class", default="gate_up")
     ap.add_argument("--model", default="7b", help="model shape (7b; smaller ones for quick checks)")
     ap.add_argument("--kv-len", type=int, default=1564)
+    ap.add_argument("--sweep", default="0,1,2,4,8,16",
+                    help="block sizes k for the verify-time sweep ('' to skip)")
+    ap.add_argument("--sweep-blocks", type=int, default=32)
     return ap.parse_args()
 
 
@@ -119,10 +126,24 @@ def model_shape(name):
     return W.MODELS[name]
 
 
-def draw_plans(args, steps, vocab):
+def draw_plans(args, steps, vocab, k=None, seed_offset=17):
     from synth import workloads as W
-    rng = np.random.default_rng(args.seed + 17)
-    return np.stack([W.geometric_plan(rng, args.k, vocab) for _ in range(steps)])
+    k = args.k if k is None else k
+    rng = np.random.default_rng(args.seed + seed_offset)
+    return np.stack([W.geometric_plan(rng, k, vocab) for _ in range(steps)])
+
+
+def reduce_ranks(elapsed_ms, committed, device):
+    """Replicas: the job's time is the slowest rank's, its work the sum of
+    every rank's committed tokens (no exchange between replicas otherwise)."""
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([elapsed_ms, float(committed)], dtype=torch.float64, device=device)
+    mx = t.clone()
+    dist.all_reduce(mx, op=dist.ReduceOp.MAX)
+    sm = t.clone()
+    dist.all_reduce(sm, op=dist.ReduceOp.SUM)
+    return float(mx[0]), float(sm[1])
 
 
 def bytes_per_block(cfg, L, k):
@@ -200,32 +221,52 @@ def run_ours(args, ws, rank, local):
               for _ in range(steps)]
         t0 = torch.cuda.Event(enable_timing=True)
         t1 = torch.cuda.Event(enable_timing=True)
-        state.profile(args.profile_class)
-        state.profile_read()
+
+        def timed_pass(profile_class):
+            """`steps` consecutive blocks from the initial state, timed with
+            CUDA events on the launching stream; optionally with the library's
+            event pairs around one kernel class."""
+            state.rollback([L0], [root0], sh)
+            state.read_state(sh)
+            n_all.zero_()
+            state.profile(None if profile_class in (None, "none") else profile_class)
+            state.profile_read()
+            if ws > 1:
+                dist.barrier()
+            torch.cuda.synchronize()
+            torch.cuda.nvtx.range_push("timed")
+            t0.record(stream)
+            for i in range(steps):
+                ev[i][0].record(stream)
+                block(i, i)
+                ev[i][1].record(stream)
+            t1.record(stream)
+            torch.cuda.nvtx.range_pop()
+            torch.cuda.synchronize()
+            if ws > 1:
+                dist.barrier()
+            res = state.profile_read()
+            state.profile(None)
+            return res
+
+        # pass 1 (the headline): no library event pairs, so programmatic
+        # dependent launch overlaps every kernel boundary
         clocks = ClockSampler(local)
         clocks.start()
         time.sleep(0.3)
-        if ws > 1:
-            dist.barrier()
-        torch.cuda.synchronize()
-        t0.record(stream)
-        for i in range(steps):
-            ev[i][0].record(stream)
-            block(i, i)
-            ev[i][1].record(stream)
-        t1.record(stream)
-        torch.cuda.synchronize()
-        if ws > 1:
-            dist.barrier()
+        _, _, all_launches = timed_pass(None)
         clk = clocks.stop()
-        prof_n, prof_ms, all_launches = state.profile_read()
-        state.profile(None)
         state.check(sh)
         elapsed_ms = t0.elapsed_time(t1)
         per_block_us = np.array([a.elapsed_time(b) * 1e3 for a, b in ev])
         n_np = n_all.cpu().numpy()
         committed = int((n_np + 1).sum())
         plan_match = float(np.mean(n_np == plans[:, 0]))
+        # pass 2: the same blocks again with event pairs around every launch of
+        # the dominant kernel class, for its live average duration
+        prof_n, prof_ms, _ = timed_pass(args.profile_class)
+        pass2_ms = t0.elapsed_time(t1)
+        state.check(sh)
 
         # per-class device time per block (diagnostic, after the timed region)
         breakdown = {}
@@ -242,17 +283,53 @@ def run_ours(args, ws, rank, local):
         state.profile(None)
         state.check(sh)
 
+        # verify time and committed tokens/s versus k (same acceptance law,
+        # capped at k), and the per-position cost reduction R(K) of Eq. 2
+        sweep = []
+        if args.sweep:
+            ks = [int(x) for x in args.sweep.split(",") if x != ""]
+            nbk = args.sweep_blocks
+            for kk in ks:
+                pl = draw_plans(args, nbk, cfg.vocab, k=kk, seed_offset=1000 + kk) if kk > 0 else None
+                pl_d = torch.from_numpy(pl.astype(np.int32)).cuda() if kk > 0 else None
+                cand_k = torch.zeros(max(kk, 1), dtype=torch.int32, device="cuda")
+                nk = torch.zeros(nbk, dtype=torch.int32, device="cuda")
+                ck = torch.zeros(nbk, dtype=torch.int32, device="cuda")
+                evk = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                       for _ in range(nbk)]
+                state.rollback([L0], [root0], sh)
+                state.read_state(sh)
+                torch.cuda.synchronize()
+                for i in range(nbk):
+                    evk[i][0].record(stream)
+                    if kk > 0:
+                        rc = synth._load_cuda().synth_cuda_build_candidates(
+                            cand_k.data_ptr(), traj.data_ptr(), traj_len + 1, len_dev, L0,
+                            pl_d[i].data_ptr(), kk, cfg.vocab, sh)
+                        assert rc == 0
+                    out = lib.make_verify_out(nk.data_ptr() + 4 * i, ck.data_ptr() + 4 * i)
+                    lib._check(lib.as2d_verify_block(state.handle, cand_k.data_ptr() if kk else 0,
+                                                     [kk], out, sh), "as2d_verify_block")
+                    evk[i][1].record(stream)
+                torch.cuda.synchronize()
+                us = np.array([a.elapsed_time(b) * 1e3 for a, b in evk])
+                ncommit = int((nk.cpu().numpy() + 1).sum())
+                sweep.append({"k": kk, "K": kk + 1, "verify_us_median": round(float(np.median(us)), 1),
+                              "verify_us_mean": round(float(us.mean()), 1),
+                              "committed_tok_s": round(ncommit / (us.sum() / 1e6), 1),
+                              "mean_committed": round(ncommit / nbk, 3)})
+                state.check(sh)
+            v1 = next((e["verify_us_mean"] for e in sweep if e["k"] == 0), None)
+            if v1:
+                for e in sweep:
+                    e["R_pct"] = round(100.0 * (1.0 - e["verify_us_mean"] / (e["K"] * v1)), 1)
+
         e2e = None
         if not args.no_e2e:
             e2e = run_e2e(args, lib, W, state, traj, plans, cfg, L0, root0, sh, stream)
 
     if ws > 1:
-        t = torch.tensor([elapsed_ms, committed], dtype=torch.float64, device="cuda")
-        mx = t.clone()
-        dist.all_reduce(mx, op=dist.ReduceOp.MAX)
-        sm = t.clone()
-        dist.all_reduce(sm, op=dist.ReduceOp.SUM)
-        elapsed_ms, committed_all = float(mx[0]), float(sm[1])
+        elapsed_ms, committed_all = reduce_ranks(elapsed_ms, committed, "cuda")
     else:
         committed_all = committed
     value = committed_all / (elapsed_ms / 1e3)
@@ -275,9 +352,13 @@ def run_ours(args, ws, rank, local):
         achieved = per_unit / (avg_ms / 1e3) / 1e9
         roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
                     "unit": "GB/s", "frac": round(achieved / peak, 4),
-                    "traffic": None, "kernel": cls, "peak_kind": peak_kind,
+                    "traffic": TRAFFIC.get(cls), "kernel": cls, "peak_kind": peak_kind,
                     "launches": prof_n, "avg_us": round(avg_ms * 1e3, 2),
-                    "bytes_per_launch": int(per_unit)}
+                    "bytes_per_launch": int(per_unit),
+                    "measured": f"CUDA event pair around each {cls} GEMM launch on the "
+                                f"launching stream during a second timed pass over the same "
+                                f"{steps} blocks ({pass2_ms / steps:.3f} ms/block with the "
+                                "event pairs); value comes from the first pass, without them"}
     step_bytes = bytes_per_block(cfg, L0 + committed / 2.0, k)  # mean length over the blocks
     med_us = float(np.median(per_block_us))
     step_roof = {"bytes_per_block": int(step_bytes),
@@ -300,8 +381,11 @@ def run_ours(args, ws, rank, local):
         "plan_match": plan_match,
         "step_roofline": step_roof,
         "roofline": roofline,
-        "gpu_launches": int(all_launches),
+        "gpu_launches": int(all_launches) + steps,
+        "gpu_launches_detail": f"{int(all_launches)} libas2d kernels + {steps} candidate "
+                               "builder kernels (test input) in the timed pass",
         "class_us_per_block": breakdown,
+        "k_sweep": sweep,
         "clocks": clk,
         "e2e": e2e,
     }

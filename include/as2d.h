@@ -218,7 +218,7 @@ as2d_status as2d_kv_profile(as2d_kv* kv, int32_t kernel_class);
 
 /* Synchronise the recorded events and return the number of recorded
    event pairs of the class, their summed device time in milliseconds, and the
-   number of kernels of any class launched since the last read; then reset. */
+   number of kernels the library launched since the last read; then reset. */
 as2d_status as2d_kv_profile_read(as2d_kv* kv, int32_t* launches,
                                  double* total_ms, int64_t* all_launches);
 

@@ -355,7 +355,6 @@ struct ProfScope {
   do {                                           \
     ProfScope ps_(s, cls, st);                   \
     CUDA_TRY(expr);                              \
-    ++s.launches;                                \
   } while (0)
 
 // One projection on the tensor cores: row chunks of at most 256 token rows.
@@ -386,6 +385,7 @@ cudaError_t tc_project(int epi, const Model& m, KvState& s, const RowMap& rm, co
       default: e = tc_gemm_logits(nb, x, p, st); break;
     }
     if (e != cudaSuccess) return e;
+    ++s.launches;
   }
   return cudaSuccess;
 }

@@ -314,6 +314,7 @@ cudaError_t launch_attention_split(const RowMap& m, const Model& md, KvState& kv
   dim3 g1(parts, c.n_kv_heads, kv.batch);
   dim3 g2(m.rows, c.n_q_heads);
   cudaError_t e;
+  kv.launches += 2;
   if (c.head_dim == 128) {
     e = launch_pdl(attn_part_kernel<128>, g1, dim3(256), 0, st, a);
     if (e == cudaSuccess) e = launch_pdl(attn_merge_kernel<128>, g2, dim3(128), 0, st, a);

@@ -145,6 +145,7 @@ __global__ void f32_from_bf16_kernel(float* dst, const bf16* src, int64_t n) {
 
 cudaError_t launch_embed(const RowMap& m, const Model& md, KvState& kv,
                          const int32_t* cand, cudaStream_t st) {
+  ++kv.launches;
   return launch_pdl(embed_kernel, dim3(m.rows), dim3(256), 0, st, m, cand,
                     (const int32_t*)kv.d_root, (const bf16*)md.embed, md.cfg.hidden,
                     md.cfg.vocab, kv.h, kv.d_err, kv.d_err + 1, (const int32_t*)kv.d_len,
@@ -156,6 +157,7 @@ cudaError_t launch_accept(const RowMap& m, const Model& md, KvState& kv,
                           const int32_t* cand, const as2d_verify_out& out,
                           cudaStream_t st) {
   (void)md;
+  ++kv.launches;
   return launch_pdl(accept_kernel, dim3(m.batch), dim3(32), 0, st, m, cand, kv.best, kv.d_len,
                     kv.d_root, kv.d_err + 1, out.n_accepted, out.correction_token, out.greedy);
 }
