@@ -35,7 +35,9 @@ WORKLOAD = "7b"
 
 # dram__bytes_read.sum + dram__bytes_write.sum per launch from one ncu capture
 # of the kernel as it stands (profiles/); None once the kernel has changed.
-TRAFFIC = {"gate_up": 276091648}  # profiles/gemm_gateup_7b_k8.md
+# dram bytes per launch from an ncu capture of the current kernel; None when
+# the kernel changed after the capture
+TRAFFIC = {"gate_up": None}
 
 
 def parse():
@@ -48,7 +50,10 @@ def parse():
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--profile-class", default="gate_up")
+    ap.add_argument("--profile-class", default="auto",
+                    help="kernel class timed live for the roofline; auto = the whole "
+                         "persistent pass when it is enabled (AS2D_PERSISTENT=1, "
+                         "k + 1 <= 32 rows), else gate_up")
     ap.add_argument("--model", default="7b", help="model shape (7b; smaller ones for quick checks)")
     ap.add_argument("--kv-len", type=int, default=1564)
     ap.add_argument("--sweep", default="0,1,2,4,8,16",
@@ -264,13 +269,16 @@ def run_ours(args, ws, rank, local):
         plan_match = float(np.mean(n_np == plans[:, 0]))
         # pass 2: the same blocks again with event pairs around every launch of
         # the dominant kernel class, for its live average duration
-        prof_n, prof_ms, _ = timed_pass(args.profile_class)
+        prof_cls = args.profile_class
+        if prof_cls == "auto":
+            prof_cls = "pass" if (k + 1) <= 32 and os.environ.get("AS2D_PERSISTENT", "0") == "1" else "gate_up"
+        prof_n, prof_ms, _ = timed_pass(prof_cls)
         pass2_ms = t0.elapsed_time(t1)
         state.check(sh)
 
         # per-class device time per block (diagnostic, after the timed region)
         breakdown = {}
-        for cls_name in ("qkv", "attention", "o", "gate_up", "down", "lm_head", "other"):
+        for cls_name in ("qkv", "attention", "o", "gate_up", "down", "lm_head", "other", "pass"):
             state.rollback([L0], [root0], sh)
             state.read_state(sh)
             state.profile(cls_name)
@@ -279,7 +287,8 @@ def run_ours(args, ws, rank, local):
             for i in range(nb_blocks):
                 block(i, i)
             n_cls, ms_cls, _ = state.profile_read()
-            breakdown[cls_name] = round(ms_cls / nb_blocks * 1e3, 1)
+            if n_cls:
+                breakdown[cls_name] = round(ms_cls / nb_blocks * 1e3, 1)
         state.profile(None)
         state.check(sh)
 
@@ -338,8 +347,10 @@ def run_ours(args, ws, rank, local):
     # roofline of the dominant kernel class (per layer: one pair of events)
     H, F = cfg.hidden, cfg.ffn
     rows = k + 1
-    cls = args.profile_class
+    cls = prof_cls
+    mean_len = L0 + committed / 2.0
     per_unit = {
+        "pass": bytes_per_block(cfg, mean_len, k),
         "gate_up": 2 * F * H * 2 + rows * (H * 4 + 2 * H * 2 + F * 2),
         "down": H * F * 2 + rows * (F * 2 + 2 * H * 4),
         "qkv": (cfg.n_q + 2 * cfg.n_kv) * cfg.head_dim * H * 2 + rows * (H * 4 + 2 * H * 2),
@@ -355,7 +366,7 @@ def run_ours(args, ws, rank, local):
                     "traffic": TRAFFIC.get(cls), "kernel": cls, "peak_kind": peak_kind,
                     "launches": prof_n, "avg_us": round(avg_ms * 1e3, 2),
                     "bytes_per_launch": int(per_unit),
-                    "measured": f"CUDA event pair around each {cls} GEMM launch on the "
+                    "measured": f"CUDA event pair around each {cls} launch on the "
                                 f"launching stream during a second timed pass over the same "
                                 f"{steps} blocks ({pass2_ms / steps:.3f} ms/block with the "
                                 "event pairs); value comes from the first pass, without them"}

@@ -208,7 +208,10 @@ as2d_status as2d_decode_step_static(as2d_model* model, void* k_cache, void* v_ca
 #define AS2D_KERNEL_DOWN 4       /* down projection + residual          */
 #define AS2D_KERNEL_LM_HEAD 5    /* final norm + LM head + argmax       */
 #define AS2D_KERNEL_OTHER 6      /* embedding gather, accept scan, ...  */
-#define AS2D_KERNEL_CLASSES 7
+#define AS2D_KERNEL_PASS 7       /* the whole pass as one persistent kernel
+                                    (opt-in: AS2D_PERSISTENT=1; calls of
+                                    at most 32 rows)                     */
+#define AS2D_KERNEL_CLASSES 8
 
 /* Record a CUDA event pair on the call's stream around the launches of
    kernel class `kernel_class` (one pair per layer, or per call for the LM

@@ -34,7 +34,7 @@ EXPORTED = ("as2d_model_load", "as2d_kv_init_prefilled", "as2d_verify_block",
             "as2d_model_free", "as2d_last_error", "as2d_kv_profile",
             "as2d_kv_profile_read", "as2d_decode_step_static")
 KERNEL_CLASSES = {"qkv": 0, "attention": 1, "o": 2, "gate_up": 3, "down": 4,
-                  "lm_head": 5, "other": 6}
+                  "lm_head": 5, "other": 6, "pass": 7}
 
 
 class as2d_config(ctypes.Structure):

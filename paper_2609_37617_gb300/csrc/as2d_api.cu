@@ -290,6 +290,7 @@ extern "C" as2d_status as2d_kv_init_prefilled(as2d_model* mh, int32_t batch,
   s.ss = cv.take<float>(R * (H / 128));
   s.ws = cv.take<float>((size_t)m.sm_count * 2 * s.nb_max * 128);
   s.counters = cv.take<int>(max_tiles);
+  s.n_counters = (int)max_tiles;
   s.attn_o = cv.take<float>(attn_rows * m.cfg.head_dim);
   s.attn_ml = cv.take<float2>(attn_rows);
   bool ok = true;
@@ -304,6 +305,13 @@ extern "C" as2d_status as2d_kv_init_prefilled(as2d_model* mh, int32_t batch,
     cudaFree(s.work);
     delete kh;
     return fail(AS2D_ERR_CUDA, "cuTensorMapEncodeTiled failed for an activation buffer");
+  }
+  e = mk_prepare(m, s);
+  if (e != cudaSuccess) {
+    cudaFree(s.mk_mem);
+    cudaFree(s.work);
+    delete kh;
+    return fail(AS2D_ERR_CUDA, std::string("preparing the persistent pass: ") + cudaGetErrorString(e));
   }
   e = cudaMemset(s.work, 0, bytes);
   if (e == cudaSuccess) e = cudaMemcpy(s.d_len, kv_len, batch * 4, cudaMemcpyHostToDevice);
@@ -321,6 +329,7 @@ extern "C" as2d_status as2d_kv_init_prefilled(as2d_model* mh, int32_t batch,
 extern "C" void as2d_kv_free(as2d_kv* kh) {
   if (!kh) return;
   for (cudaEvent_t e : kh->s.prof_events) cudaEventDestroy(e);
+  cudaFree(kh->s.mk_mem);
   cudaFree(kh->s.work);
   delete kh;
 }
@@ -385,7 +394,7 @@ cudaError_t tc_project(int epi, const Model& m, KvState& s, const RowMap& rm, co
       default: e = tc_gemm_logits(nb, x, p, st); break;
     }
     if (e != cudaSuccess) return e;
-    ++s.launches;
+    s.launches += 1;
   }
   return cudaSuccess;
 }
@@ -414,7 +423,15 @@ as2d_status run_block(KvState& s, const int32_t* cand, const int32_t* k,
 
   // One pass of the verification step (Section 3.2; App. C.2): embedding
   // gather, n_layers x {QKV + RoPE + KV append, attention, O + residual,
-  // gate/up + SwiGLU, down + residual}, LM head + argmax, accept scan.
+  // gate/up + SwiGLU, down + residual}, LM head + argmax, accept scan, as a
+  // sequence of kernels chained by programmatic dependent launch.  With
+  // AS2D_PERSISTENT=1 in the environment, calls of at most 32 rows run it as
+  // one persistent kernel instead (same arithmetic, same results).
+  if (mk_usable(s, rm.rows)) {
+    LAUNCH(AS2D_KERNEL_PASS, launch_mk(rm, m, s, cand, *out, st));
+    for (int b = 0; b < s.batch; ++b) s.len_upper[b] += (k ? k[b] : 0) + 1;
+    return AS2D_OK;
+  }
   LAUNCH(AS2D_KERNEL_OTHER, launch_embed(rm, m, s, cand, st));
   TcParams tp{};
   tp.h = s.h;
@@ -525,6 +542,9 @@ extern "C" as2d_status as2d_kv_check(as2d_kv* kh, void* stream) {
   if (err != 0) {
     int32_t zero = 0;
     CUDA_TRY(cudaMemcpy(kh->s.d_err, &zero, 4, cudaMemcpyHostToDevice));
+    // a kernel that gave up may have left split-tile arrival counts behind
+    if (kh->s.counters && kh->s.n_counters > 0)
+      CUDA_TRY(cudaMemset(kh->s.counters, 0, (size_t)kh->s.n_counters * 4));
     std::string msg = "device error:";
     if (err & kErrBadToken) msg += " candidate or root token outside [0, vocab);";
     if (err & kErrRollback) msg += " rollback beyond the committed length;";

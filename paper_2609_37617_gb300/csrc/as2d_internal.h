@@ -155,6 +155,7 @@ struct KvState {
   int nb_max = 16;
   float* ws = nullptr;       // [sm_count][2][nb_max][128] partial GEMM tiles
   int* counters = nullptr;   // [max tiles] stream-K arrival counters
+  int n_counters = 0;
   float* ss = nullptr;       // [hidden / 128][rows_alloc] partial sums of h^2
   float* attn_o = nullptr;   // [batch][n_kv][parts][qmax][d] attention partials
   float2* attn_ml = nullptr; // [batch][n_kv][parts][qmax] (max, sum) base 2
@@ -162,6 +163,12 @@ struct KvState {
   int attn_qmax = 0;         // (kMaxK + 1) * group, rounded up to 16
   // TMA descriptors of the activation operands, per token-row padding
   CUtensorMap tm_xn[kNbCount], tm_ao[kNbCount], tm_u[kNbCount];
+  // persistent single-launch pass (k_mk.cu)
+  bool mk_ok = false;
+  void* mk_mem = nullptr;          // phase table, then per-phase arrival counters
+  unsigned int* mk_bar = nullptr;
+  int mk_n_phases = 0;
+  unsigned int mk_gen = 0;         // calls so far
   // measurement support
   int prof_class = -1;
   std::vector<cudaEvent_t> prof_events;  // pairs
@@ -186,6 +193,12 @@ cudaError_t pack_weights(bf16* dst, int n_rows, int K, const void* const* segs,
 int attn_partitions(int capacity);
 cudaError_t launch_attention_split(const RowMap& m, const Model& md, KvState& kv, int layer,
                                    cudaStream_t st);
+
+// Persistent single-launch pass for calls of at most 32 rows (k_mk.cu).
+cudaError_t mk_prepare(const Model& m, KvState& kv);
+bool mk_usable(const KvState& kv, int rows);
+cudaError_t launch_mk(const RowMap& rm, const Model& m, KvState& kv, const int32_t* cand,
+                      const as2d_verify_out& out, cudaStream_t st);
 
 // Tensor-core GEMM launchers (k_tc_*.cu), one per fused epilogue.
 cudaError_t tc_gemm_qkv(int nb, const CUtensorMap& x, const TcParams& p,

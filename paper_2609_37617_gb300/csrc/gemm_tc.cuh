@@ -21,10 +21,12 @@
 //     fp32 accumulator from TMEM (double-buffered);
 //   * stream-K: the (tile, 64-column k-block) units are split evenly over a
 //     persistent grid of one CTA per SM, so every SM streams the same number
-//     of weight bytes whatever N is.  A tile cut between CTAs is finished by
-//     the last CTA to arrive (an arrival counter, no waiting), which adds the
-//     partial tiles in CTA order: the sum order depends on (N, K, grid) only,
-//     never on the number of token rows, so results are batch invariant;
+//     of weight bytes whatever N is.  A CTA that holds a whole tile applies
+//     the epilogue itself; each CTA that holds part of a tile cut between
+//     CTAs stores its partial tile, and the last of them to arrive (an atomic
+//     count per tile) adds the parts in CTA order and applies the epilogue:
+//     the sum order depends on (N, K, grid) only, never on the number of
+//     token rows or on arrival order, so results are batch invariant;
 //   * the epilogue is fused: RoPE + KV-cache append (QKV), residual add
 //     (O, down), SwiGLU (gate/up), and logits + argmax (LM head).
 // Every mbarrier wait is bounded in time; on expiry the kernel records an
@@ -60,7 +62,7 @@ struct TcShape {
   static constexpr int NBUF = 2 * ACC_COLS <= 512 ? 2 : 1;
   static constexpr uint32_t TMEM_COLS = (NBUF * ACC_COLS < 32) ? 32 : NBUF * ACC_COLS;
   static constexpr uint32_t SMEM =
-      1024 + S * (A_BYTES + STAGE_B) + 128 * SP * 4 + (NB + 64) * 4 + (2 * S + 5) * 8 + 16;
+      1024 + S * (A_BYTES + STAGE_B) + 128 * SP * 4 + (3 * NB + 64) * 4 + (2 * S + 5) * 8 + 16;
 };
 
 __device__ __forceinline__ float tc_silu(float x) { return x / (1.0f + expf(-x)); }
@@ -78,24 +80,56 @@ __device__ __forceinline__ int tc_owner(long long u, const TcParams& p) {
   return (int)(((u + 1) * (long long)p.grid - 1) / p.units);
 }
 
-// Fused epilogue of one 16-row chunk: sC[n * SP + j] holds D for tile row n
-// and token row row0 + m0 + j.  Runs on the 128 epilogue threads (et).
+// Operands of one 16-row epilogue chunk that come from memory (the residual
+// and the norm gain for RESID, the rotary table for QKV), fetched by
+// tc_epilogue_load before they are needed so that their loads overlap other
+// loads of the caller.
+struct TcEpiIn {
+  float hv[16];
+  float gn;
+  float2 cs[16];
+};
+
 template <int NB, int EPI>
-__device__ __forceinline__ void tc_epilogue_chunk(const TcParams& p, const float* sC, float* red,
-                                                  int tile, int m0, int et) {
+__device__ __forceinline__ void tc_epilogue_load(const TcParams& p, TcEpiIn& in, int tile, int m0,
+                                                 int et) {
+  constexpr int CH = TcShape<NB>::CH;
+  const int n = et, col = tile * 128 + n;
+  if (EPI == TC_RESID) {
+    in.gn = p.g_next[col];
+#pragma unroll
+    for (int j = 0; j < CH; ++j)
+      if (m0 + j < p.rows) in.hv[j] = p.h[(size_t)(p.row0 + m0 + j) * p.N + col];
+  } else if (EPI == TC_QKV) {
+    const int d = p.d, half = d >> 1;
+    const int head = col / d, e = col - head * d;
+    const int i = e < half ? e : e - half;
+    if (head < p.nq + p.nkv) {
+#pragma unroll
+      for (int j = 0; j < CH; ++j)
+        if (m0 + j < p.rows) in.cs[j] = p.rope[(size_t)(p.row0 + m0 + j) * half + i];
+    }
+  }
+}
+
+// Fused epilogue of one 16-row chunk: sC[n * SP + j] holds D for tile row n
+// and token row row0 + m0 + j; `in` holds the chunk's tc_epilogue_load.  Runs
+// on the 128 epilogue threads (et).
+template <int NB, int EPI>
+__device__ __forceinline__ void tc_epilogue_apply(const TcParams& p, const TcEpiIn& in,
+                                                  const float* sC, float* red, const int* s_pos,
+                                                  const int* s_req, int tile, int m0, int et) {
   constexpr int SP = TcShape<NB>::SP;
   constexpr int CH = TcShape<NB>::CH;
   if (EPI == TC_RESID) {
-    // thread et owns tile row n = et for the chunk's 16 token rows: all
-    // residual loads are issued before any add, so they overlap.  The new
+    // thread et owns tile row n = et for the chunk's 16 token rows.  The new
     // residual also yields the next projection's operand and its share of
     // the row's sum of squares (warp butterflies, then warps in order).
     const int n = et, col = tile * 128 + n;
-    const float gn = p.g_next[col];
+    const float gn = in.gn;
     float hv[CH];
 #pragma unroll
-    for (int j = 0; j < CH; ++j)
-      if (m0 + j < p.rows) hv[j] = p.h[(size_t)(p.row0 + m0 + j) * p.N + col];
+    for (int j = 0; j < CH; ++j) hv[j] = in.hv[j];
 #pragma unroll
     for (int j = 0; j < CH; ++j) {
       if (m0 + j < p.rows) {
@@ -135,36 +169,38 @@ __device__ __forceinline__ void tc_epilogue_chunk(const TcParams& p, const float
       p.u[at + (size_t)p.lo_row * F] = __float2bfloat16_rn(uv - __bfloat162float(uh));
     }
   } else if (EPI == TC_QKV) {
+    // thread et owns tile row n = et (one element of one head) for the chunk's
+    // 16 token rows
     const int d = p.d, half = d >> 1, q_dim = p.nq * d;
-    for (int idx = et; idx < 128 * CH; idx += 128) {
-      const int j = idx >> 7, n = idx & 127, m = m0 + j;
+    const int n = et, col = tile * 128 + n, head = col / d, e = col - head * d;
+    const int partner = e < half ? n + half : n - half;
+    const bool rotate = head < p.nq + p.nkv;
+    const float2* cs = in.cs;
+    int pos[CH];
+#pragma unroll
+    for (int j = 0; j < CH; ++j)
+      if (m0 + j < p.rows) pos[j] = s_pos[m0 + j];
+#pragma unroll
+    for (int j = 0; j < CH; ++j) {
+      const int m = m0 + j;
       if (m >= p.rows) break;
       const int gm = p.row0 + m;
-      const int col = tile * 128 + n, head = col / d, e = col - head * d;
       const float x = sC[n * SP + j];
-      if (head < p.nq + p.nkv) {
-        const int i = e < half ? e : e - half;
-        const float2 cs = p.rope[(size_t)gm * half + i];
-        float y;
-        if (e < half) {
-          y = x * cs.x - sC[(n + half) * SP + j] * cs.y;
-        } else {
-          y = x * cs.x + sC[(n - half) * SP + j] * cs.y;
-        }
+      if (rotate) {
+        const float xp = sC[partner * SP + j];
+        const float y = (e < half) ? x * cs[j].x - xp * cs[j].y : x * cs[j].x + xp * cs[j].y;
         if (head < p.nq) {
           p.q[(size_t)gm * q_dim + col] = y;
         } else {
-          const int b = row_request(p.rm, gm);
-          const int pos = p.len[b] + (gm - p.rm.start[b]);
+          const int b = s_req[m];
           const size_t off =
-              ((((size_t)p.layer * p.batch + b) * p.nkv + (head - p.nq)) * p.cap + pos) * d + e;
+              ((((size_t)p.layer * p.batch + b) * p.nkv + (head - p.nq)) * p.cap + pos[j]) * d + e;
           p.kc[off] = __float2bfloat16_rn(y);
         }
       } else {
-        const int b = row_request(p.rm, gm);
-        const int pos = p.len[b] + (gm - p.rm.start[b]);
+        const int b = s_req[m];
         const size_t off =
-            ((((size_t)p.layer * p.batch + b) * p.nkv + (head - p.nq - p.nkv)) * p.cap + pos) * d + e;
+            ((((size_t)p.layer * p.batch + b) * p.nkv + (head - p.nq - p.nkv)) * p.cap + pos[j]) * d + e;
         p.vc[off] = __float2bfloat16_rn(x);
       }
     }
@@ -200,6 +236,15 @@ __device__ __forceinline__ void tc_epilogue_chunk(const TcParams& p, const float
   }
 }
 
+template <int NB, int EPI>
+__device__ __forceinline__ void tc_epilogue_chunk(const TcParams& p, const float* sC, float* red,
+                                                  const int* s_pos, const int* s_req, int tile,
+                                                  int m0, int et) {
+  TcEpiIn in;
+  tc_epilogue_load<NB, EPI>(p, in, tile, m0, et);
+  tc_epilogue_apply<NB, EPI>(p, in, sC, red, s_pos, s_req, tile, m0, et);
+}
+
 // 16 accumulator columns of chunk ch for this thread's TMEM lane: the hi and
 // lo results are added here (hi + lo, fixed order).
 template <int NB>
@@ -210,6 +255,109 @@ __device__ __forceinline__ void tc_load_acc(uint32_t tbase, int ch, uint32_t (&v
   ptx::tmem_ld_wait();
 #pragma unroll
   for (int j = 0; j < 16; ++j) v[j] = __float_as_uint(__uint_as_float(v[j]) + __uint_as_float(w[j]));
+}
+
+// Per-row values the epilogue needs, for the launch's token rows: 1 / rms of
+// each row from the producer's per-tile sums of squares (in tile order), and
+// for QKV the request and cache position of each row.  Run by the 128
+// epilogue threads (et), ends with their named barrier.
+template <int NB, int EPI>
+__device__ __forceinline__ void tc_row_prologue(const TcParams& p, float* s_rinv, int* s_pos,
+                                                int* s_req, int et) {
+    // every load below is issued before any result is used: one memory
+    // round trip for up to 32 tiles' sums (hidden <= 4096)
+    for (int m = et; m < p.rows; m += 128) {
+      const int gm = p.row0 + m;
+      int len_b = 0, b = 0;
+      if (EPI == TC_QKV) {
+        b = row_request(p.rm, gm);
+        len_b = p.len[b];
+      }
+      if (EPI != TC_RESID) {
+        // 1 / rms of the token row from the producer's per-tile sums (in order)
+        const float* src = p.ss + gm;
+        float tot = 0.f;
+        for (int t0 = 0; t0 < p.n_htiles; t0 += 32) {
+          float v[32];
+#pragma unroll
+          for (int u = 0; u < 32; ++u)
+            v[u] = (t0 + u < p.n_htiles) ? src[(size_t)(t0 + u) * p.ss_ld] : 0.f;
+#pragma unroll
+          for (int u = 0; u < 32; ++u) tot += v[u];
+        }
+        s_rinv[m] = rsqrtf(tot / (float)p.hidden + p.eps);
+      }
+      if (EPI == TC_QKV) {
+        s_req[m] = b;
+        s_pos[m] = len_b + (gm - p.rm.start[b]);
+      }
+    }
+    if (EPI != TC_RESID) ptx::named_bar_sync(1, 128);
+}
+
+// Adds the partial tiles of a split tile (parts c_first .. c_first + nparts - 1
+// in CTA order, all parts' loads issued at once), scales like the GEMM's own
+// epilogue and applies the fused epilogue.  128 threads (nl = tile row, et),
+// named barrier 1; sC, s_rinv, red, s_pos, s_req as in the GEMM epilogue;
+// PROLOGUE: also fills s_rinv, s_pos, s_req (tc_row_prologue), its loads
+// overlapping the parts' loads.
+template <int NB, int EPI, int MAXP = 8, bool PROLOGUE = false>
+__device__ __forceinline__ void tc_reduce_tile(const TcParams& p, float* sC, float* s_rinv,
+                                               float* red, int* s_pos, int* s_req,
+                                               int tile, int c_first, int nparts, int nl, int et) {
+  // MAXP parts are in flight at a time; the parts are added in CTA order
+  // whatever MAXP is, so it does not change the result.  The first parts, the
+  // epilogue's operands and (PROLOGUE) the row prologue's loads are all
+  // issued before any of them is used.
+  using Sh = TcShape<NB>;
+  constexpr int CH = Sh::CH, SP = Sh::SP;
+  const int nchunks = (p.rows + CH - 1) / CH;
+  for (int ch = 0; ch < nchunks; ++ch) {
+    const int live = p.rows - ch * CH;
+    float acc[CH];
+#pragma unroll
+    for (int j = 0; j < CH; ++j) acc[j] = 0.f;
+    TcEpiIn in;
+    for (int part0 = 0; part0 < nparts; part0 += MAXP) {
+      float4 v[MAXP][4];
+#pragma unroll
+      for (int pp = 0; pp < MAXP; ++pp) {
+        if (part0 + pp < nparts) {
+          const int cp = c_first + part0 + pp;
+          // slot 1 holds a CTA's last segment when it began in an earlier tile
+          const int sl = (cp == c_first && (int)(tc_start(cp, p) / p.kb) != tile) ? 1 : 0;
+          const float* src = p.ws + ((size_t)(cp * 2 + sl) * 128 + nl) * NB + ch * CH;
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+            if (4 * q < live) v[pp][q] = __ldcg(reinterpret_cast<const float4*>(src) + q);
+        }
+      }
+      if (part0 == 0) {
+        tc_epilogue_load<NB, EPI>(p, in, tile, ch * CH, et);
+        if (PROLOGUE && ch == 0) tc_row_prologue<NB, EPI>(p, s_rinv, s_pos, s_req, et);
+      }
+#pragma unroll
+      for (int pp = 0; pp < MAXP; ++pp) {
+        if (part0 + pp < nparts) {
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            if (4 * q < live) {
+              acc[4 * q] += v[pp][q].x;
+              acc[4 * q + 1] += v[pp][q].y;
+              acc[4 * q + 2] += v[pp][q].z;
+              acc[4 * q + 3] += v[pp][q].w;
+            }
+          }
+        }
+      }
+    }
+    ptx::named_bar_sync(1, 128);
+#pragma unroll
+    for (int j = 0; j < CH; ++j)
+      sC[nl * SP + j] = (EPI == TC_RESID) ? acc[j] : acc[j] * s_rinv[ch * CH + j];
+    ptx::named_bar_sync(1, 128);
+    tc_epilogue_apply<NB, EPI>(p, in, sC, red, s_pos, s_req, tile, ch * CH, et);
+  }
 }
 
 template <int NB, int EPI>
@@ -232,7 +380,9 @@ __global__ void __launch_bounds__(192, 1)
   float* sC = reinterpret_cast<float*>(sB + S * STAGE_B);
   float* s_rinv = sC + 128 * SP;  // [NB] 1 / rms of each token row (normed inputs)
   float* red = s_rinv + NB;       // [64] cross-warp reduction scratch
-  uint64_t* full = reinterpret_cast<uint64_t*>(red + 64);
+  int* s_pos = reinterpret_cast<int*>(red + 64);  // [NB] cache position of each token row
+  int* s_req = s_pos + NB;                        // [NB] request of each token row
+  uint64_t* full = reinterpret_cast<uint64_t*>(s_req + NB);
   uint64_t* empty = full + S;
   uint64_t* acc_full = empty + S;   // [2]
   uint64_t* acc_empty = acc_full + 2;  // [2]
@@ -313,6 +463,7 @@ __global__ void __launch_bounds__(192, 1)
       for (int j = (it > S ? it - S : 0); j < it; ++j)
         ptx::mbar_wait(&full[j % S], (uint32_t)(j / S) & 1u, p.timeout_ns);
     }
+    __syncwarp();  // lanes 1..31 wait for lane 0: the warp reaches the barrier converged
   } else if (warp == 1) {
     // ---------------- MMA issuer ----------------
     if (lane == 0) {
@@ -367,29 +518,14 @@ __global__ void __launch_bounds__(192, 1)
       ptx::mma_commit(drain);
       ptx::mbar_wait(drain, 0, p.timeout_ns);
     }
+    __syncwarp();
   } else {
     // ---------------- epilogue: warps 2..5, one TMEM lane each ----------------
     ptx::griddep_wait();  // the epilogue reads and writes the predecessors' outputs
     const int q4 = warp & 3;
     const int nl = q4 * 32 + lane;  // tile row this thread drains
     const int et = threadIdx.x - 64;
-    if (EPI != TC_RESID) {
-      // 1 / rms of each token row from the producer's per-tile sums (in order)
-      for (int m = et; m < p.rows; m += 128) {
-        const float* src = p.ss + p.row0 + m;
-        float tot = 0.f;
-        for (int t0 = 0; t0 < p.n_htiles; t0 += 8) {
-          float v[8];
-#pragma unroll
-          for (int u = 0; u < 8; ++u)
-            v[u] = (t0 + u < p.n_htiles) ? src[(size_t)(t0 + u) * p.ss_ld] : 0.f;
-#pragma unroll
-          for (int u = 0; u < 8; ++u) tot += v[u];
-        }
-        s_rinv[m] = rsqrtf(tot / (float)p.hidden + p.eps);
-      }
-      ptx::named_bar_sync(1, 128);
-    }
+    tc_row_prologue<NB, EPI>(p, s_rinv, s_pos, s_req, et);
     const int nchunks = (p.rows + CH - 1) / CH;
     const int first_tile = (int)(u0 / p.kb);
     int seg = 0;
@@ -400,9 +536,9 @@ __global__ void __launch_bounds__(192, 1)
       const bool whole = (u == tstart && send == tend);
       const int buf = seg % NBUF;
       const uint32_t bph = (uint32_t)(seg / NBUF) & 1u;
-      if (!ptx::mbar_wait(&acc_full[buf], bph, p.timeout_ns)) {
-        atomicOr(p.err, kErrTimeout);
-        break;
+      if (!ptx::group_all(ptx::mbar_wait(&acc_full[buf], bph, p.timeout_ns), 1, 128)) {
+        if (et == 0) atomicOr(p.err, kErrTimeout);
+        break;  // every epilogue thread leaves together
       }
       ptx::tc_fence_after();
       const uint32_t tbase = tmem + (uint32_t)(buf * ACC_COLS) + ((uint32_t)(q4 * 32) << 16);
@@ -416,7 +552,7 @@ __global__ void __launch_bounds__(192, 1)
             sC[nl * SP + j] = (EPI == TC_RESID) ? __uint_as_float(v[j])
                                                 : __uint_as_float(v[j]) * s_rinv[ch * CH + j];
           ptx::named_bar_sync(1, 128);
-          tc_epilogue_chunk<NB, EPI>(p, sC, red, tile, ch * CH, et);
+          tc_epilogue_chunk<NB, EPI>(p, sC, red, s_pos, s_req, tile, ch * CH, et);
         }
         ptx::tc_fence_before();
         __syncwarp();
@@ -437,57 +573,20 @@ __global__ void __launch_bounds__(192, 1)
         ptx::tc_fence_before();
         __syncwarp();
         if (lane == 0) ptx::mbar_arrive(&acc_empty[buf]);
+        // the last CTA to store a part of this tile adds the parts, in CTA
+        // order whichever CTA that is, and applies the epilogue
         __threadfence();
         ptx::named_bar_sync(1, 128);
         const int c_first = tc_owner(tstart, p), c_last = tc_owner(tend - 1, p);
         const int nparts = c_last - c_first + 1;
         if (et == 0) flags[1] = (atomicAdd(&p.counters[tile], 1) == nparts - 1) ? 1 : 0;
         ptx::named_bar_sync(1, 128);
-        if (flags[1]) {
+        const int last = flags[1];
+        ptx::named_bar_sync(1, 128);
+        if (last) {
           __threadfence();
-          for (int ch = 0; ch < nchunks; ++ch) {
-            // partial tiles added in CTA order; each part's 16 loads are
-            // independent, so a part costs one round trip to L2
-            float acc[CH];
-#pragma unroll
-            for (int j = 0; j < CH; ++j) acc[j] = 0.f;
-            const int live = p.rows - ch * CH;  // token rows of this chunk that exist
-            for (int part0 = 0; part0 < nparts; part0 += 4) {
-              float4 v[4][4];
-#pragma unroll
-              for (int pp = 0; pp < 4; ++pp) {
-                if (part0 + pp < nparts) {
-                  const int cp = c_first + part0 + pp;
-                  const int sl = ((int)(tc_start(cp, p) / p.kb) == tile) ? 0 : 1;
-                  const float* src = p.ws + ((size_t)(cp * 2 + sl) * 128 + nl) * NB + ch * CH;
-#pragma unroll
-                  for (int q = 0; q < 4; ++q)
-                    if (4 * q < live) v[pp][q] = __ldcg(reinterpret_cast<const float4*>(src) + q);
-                }
-              }
-#pragma unroll
-              for (int pp = 0; pp < 4; ++pp) {
-                if (part0 + pp < nparts) {
-#pragma unroll
-                  for (int q = 0; q < 4; ++q) {
-                    if (4 * q < live) {
-                      acc[4 * q] += v[pp][q].x;
-                      acc[4 * q + 1] += v[pp][q].y;
-                      acc[4 * q + 2] += v[pp][q].z;
-                      acc[4 * q + 3] += v[pp][q].w;
-                    }
-                  }
-                }
-              }
-            }
-            ptx::named_bar_sync(1, 128);
-#pragma unroll
-            for (int j = 0; j < CH; ++j)
-              sC[nl * SP + j] = (EPI == TC_RESID) ? acc[j] : acc[j] * s_rinv[ch * CH + j];
-            ptx::named_bar_sync(1, 128);
-            tc_epilogue_chunk<NB, EPI>(p, sC, red, tile, ch * CH, et);
-          }
-          if (et == 0) p.counters[tile] = 0;
+          tc_reduce_tile<NB, EPI, 6>(p, sC, s_rinv, red, s_pos, s_req, tile, c_first, nparts, nl, et);
+          if (et == 0) p.counters[tile] = 0;  // ready for the next launch
         }
       }
       u = send;
