@@ -265,6 +265,9 @@ extern "C" as2d_status as2d_kv_init_prefilled(as2d_model* mh, int32_t batch,
            align_up(2 * R * m.q_dim * 2, 256) + align_up(2 * R * F * 2, 256) + align_up(R * 8, 256) +
            align_up(R * (m.cfg.head_dim / 2) * 8, 256) + align_up(R * (H / 128) * 4, 256) +
            align_up((size_t)m.sm_count * 2 * s.nb_max * 128 * 4, 256) + align_up(max_tiles * 4, 256);
+  s.qkv_split = qkv_split_for(m);
+  const size_t qkv_tiles = (size_t)(m.qkv_rows + 127) / 128;
+  bytes += align_up(qkv_tiles * s.qkv_split * R * 128 * 4, 256) + align_up(R * 4, 256);
   const int group = m.cfg.n_q_heads / m.cfg.n_kv_heads;
   s.attn_parts = attn_partitions(capacity);
   s.attn_qmax = ((kMaxK + 1) * group + 15) / 16 * 16;
@@ -291,6 +294,8 @@ extern "C" as2d_status as2d_kv_init_prefilled(as2d_model* mh, int32_t batch,
   s.ws = cv.take<float>((size_t)m.sm_count * 2 * s.nb_max * 128);
   s.counters = cv.take<int>(max_tiles);
   s.n_counters = (int)max_tiles;
+  s.qkv_part = cv.take<float>(qkv_tiles * s.qkv_split * R * 128);
+  s.qkv_rinv = cv.take<float>(R);
   s.attn_o = cv.take<float>(attn_rows * m.cfg.head_dim);
   s.attn_ml = cv.take<float2>(attn_rows);
   bool ok = true;
@@ -367,6 +372,21 @@ struct ProfScope {
   } while (0)
 
 // One projection on the tensor cores: row chunks of at most 256 token rows.
+}  // namespace
+
+// CTAs per tile of the QKV projection's K split: as many as fill the SMs
+// (at most 8 and at most one per 64-column block).  Depends on the model and
+// the device only.
+int as2d::qkv_split_for(const Model& m) {
+  const int tiles = (m.qkv_rows + 127) / 128, kb = m.cfg.hidden / 64;
+  int s = m.sm_count / tiles;
+  if (s > 8) s = 8;
+  if (s > kb) s = kb;
+  return s < 1 ? 1 : s;
+}
+
+namespace {
+
 cudaError_t tc_project(int epi, const Model& m, KvState& s, const RowMap& rm, const bf16* w,
                        const CUtensorMap* xmaps, int N, int K, TcParams p, cudaStream_t st) {
   p.w = w;
@@ -376,6 +396,14 @@ cudaError_t tc_project(int epi, const Model& m, KvState& s, const RowMap& rm, co
   p.kb = (K + 63) / 64;
   p.units = (long long)p.n_tiles * p.kb;
   p.grid = (int)(p.units < m.sm_count ? p.units : m.sm_count);
+  p.split = 0;
+  if (epi == TC_PART) {
+    p.split = s.qkv_split;
+    p.grid = p.n_tiles * p.split;
+    p.part = s.qkv_part;
+    p.part_rinv = s.qkv_rinv;
+    p.part_ld = s.rows_alloc;
+  }
   p.ws = s.ws;
   p.counters = s.counters;
   p.err = s.d_err;
@@ -389,6 +417,7 @@ cudaError_t tc_project(int epi, const Model& m, KvState& s, const RowMap& rm, co
     cudaError_t e;
     switch (epi) {
       case TC_QKV: e = tc_gemm_qkv(nb, x, p, st); break;
+      case TC_PART: e = tc_gemm_part(nb, x, p, st); break;
       case TC_RESID: e = tc_gemm_resid(nb, x, p, st); break;
       case TC_SWIGLU: e = tc_gemm_swiglu(nb, x, p, st); break;
       default: e = tc_gemm_logits(nb, x, p, st); break;
@@ -422,7 +451,7 @@ as2d_status run_block(KvState& s, const int32_t* cand, const int32_t* k,
   const as2d_config& c = m.cfg;
 
   // One pass of the verification step (Section 3.2; App. C.2): embedding
-  // gather, n_layers x {QKV + RoPE + KV append, attention, O + residual,
+  // gather, n_layers x {QKV (split-K sums), RoPE + KV append + attention, O + residual,
   // gate/up + SwiGLU, down + residual}, LM head + argmax, accept scan, as a
   // sequence of kernels chained by programmatic dependent launch.  With
   // AS2D_PERSISTENT=1 in the environment, calls of at most 32 rows run it as
@@ -458,7 +487,7 @@ as2d_status run_block(KvState& s, const int32_t* cand, const int32_t* k,
   const int H = c.hidden, F = c.ffn;
   for (int l = 0; l < c.n_layers; ++l) {
     tp.layer = l;
-    LAUNCH(AS2D_KERNEL_QKV, tc_project(TC_QKV, m, s, rm, m.w_qkv[l], s.tm_xn, m.qkv_rows, H, tp, st));
+    LAUNCH(AS2D_KERNEL_QKV, tc_project(TC_PART, m, s, rm, m.w_qkv[l], s.tm_xn, m.qkv_rows, H, tp, st));
     LAUNCH(AS2D_KERNEL_ATTENTION, launch_attention_split(rm, m, s, l, st));
     tp.g_next = m.mlp_norm[l];
     LAUNCH(AS2D_KERNEL_O, tc_project(TC_RESID, m, s, rm, m.w_o[l], s.tm_ao, H, m.q_dim, tp, st));
@@ -622,8 +651,11 @@ constexpr size_t kOffCnt = kOffWs + sa((size_t)kStaticMaxSms * 2 * 16 * 128 * 4)
 constexpr size_t kOffAttnO = kOffCnt + sa((size_t)(kStaticMaxVocab / 128 + 64) * 4);
 constexpr size_t kOffAttnMl =
     kOffAttnO + sa((size_t)kStaticMaxKvHeads * kStaticParts * kStaticMaxGroup * 128 * 4);
-constexpr size_t kStaticScratchBytes =
+constexpr size_t kStaticMaxQkvTiles = (kStaticMaxQDim + 2 * kStaticMaxKvHeads * 128) / 128;
+constexpr size_t kOffQkvPart =
     kOffAttnMl + sa((size_t)kStaticMaxKvHeads * kStaticParts * kStaticMaxGroup * 8);
+constexpr size_t kOffQkvRinv = kOffQkvPart + sa(kStaticMaxQkvTiles * 8 * kStaticRows * 128 * 4);
+constexpr size_t kStaticScratchBytes = kOffQkvRinv + sa((size_t)kStaticRows * 4);
 
 struct StaticDevice {
   bool ready = false;
@@ -715,6 +747,9 @@ extern "C" as2d_status as2d_decode_step_static(as2d_model* mh, void* k_cache, vo
   s.counters = (int*)(b + kOffCnt);
   s.attn_o = (float*)(b + kOffAttnO);
   s.attn_ml = (float2*)(b + kOffAttnMl);
+  s.qkv_part = (float*)(b + kOffQkvPart);
+  s.qkv_rinv = (float*)(b + kOffQkvRinv);
+  s.qkv_split = qkv_split_for(m);
   s.attn_parts = (capacity + 63) / 64;
   s.attn_qmax = ((c.n_q_heads / c.n_kv_heads) + 15) / 16 * 16;
   s.tm_xn[0] = sd.tm_xn;
@@ -759,7 +794,7 @@ extern "C" as2d_status as2d_decode_step_static(as2d_model* mh, void* k_cache, vo
   tp.hidden = c.hidden;
   for (int l = 0; l < c.n_layers; ++l) {
     tp.layer = l;
-    LAUNCH(AS2D_KERNEL_QKV, tc_project(TC_QKV, m, s, rm, m.w_qkv[l], s.tm_xn, m.qkv_rows, H, tp, st));
+    LAUNCH(AS2D_KERNEL_QKV, tc_project(TC_PART, m, s, rm, m.w_qkv[l], s.tm_xn, m.qkv_rows, H, tp, st));
     LAUNCH(AS2D_KERNEL_ATTENTION, launch_attention_split(rm, m, s, l, st));
     tp.g_next = m.mlp_norm[l];
     LAUNCH(AS2D_KERNEL_O, tc_project(TC_RESID, m, s, rm, m.w_o[l], s.tm_ao, H, m.q_dim, tp, st));
@@ -772,4 +807,4 @@ extern "C" as2d_status as2d_decode_step_static(as2d_model* mh, void* k_cache, vo
   return AS2D_OK;
 }
 
-static_assert(kStaticScratchBytes == 9784064, "as2d.h states the fixed working-memory size");
+static_assert(kStaticScratchBytes == 12930048, "as2d.h states the fixed working-memory size");

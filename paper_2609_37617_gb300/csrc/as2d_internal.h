@@ -42,7 +42,7 @@ enum : int32_t {
   kErrTimeout = 4,
 };
 
-enum TcEpi { TC_QKV = 0, TC_RESID = 1, TC_SWIGLU = 2, TC_LOGITS = 3 };
+enum TcEpi { TC_QKV = 0, TC_RESID = 1, TC_SWIGLU = 2, TC_LOGITS = 3, TC_PART = 4 };
 
 struct TcParams {
   const bf16* w;         // packed weight blocks (k_pack.cu), unit u at u * 8192
@@ -50,7 +50,11 @@ struct TcParams {
   int N, K;              // logical W is [N][K]
   int n_tiles, kb;       // 128-row tiles, 64-column k-blocks
   long long units;       // n_tiles * kb
-  int grid;              // CTAs (persistent)
+  int grid;              // CTAs
+  int split;             // TC_PART: CTAs per tile (K split), else 0 (stream-K)
+  float* part;           // TC_PART: [tile][split][part_ld][128] fp32 sums
+  float* part_rinv;      // TC_PART: [part_ld] 1 / rms of each token row
+  int part_ld;           // rows_alloc
   int rows;              // token rows handled by this launch
   int row0;              // first token row of this launch
   float* ws;             // [grid][2][NB][128] partial tiles
@@ -154,6 +158,9 @@ struct KvState {
   int rows_alloc = 0;        // activation rows allocated (>= every NB used)
   int nb_max = 16;
   float* ws = nullptr;       // [sm_count][2][nb_max][128] partial GEMM tiles
+  float* qkv_part = nullptr;   // [qkv tiles][qkv_split][rows_alloc][128] split-K sums
+  float* qkv_rinv = nullptr;   // [rows_alloc] 1 / rms of each row at the QKV projection
+  int qkv_split = 1;
   int* counters = nullptr;   // [max tiles] stream-K arrival counters
   int n_counters = 0;
   float* ss = nullptr;       // [hidden / 128][rows_alloc] partial sums of h^2
@@ -201,6 +208,8 @@ cudaError_t launch_mk(const RowMap& rm, const Model& m, KvState& kv, const int32
                       const as2d_verify_out& out, cudaStream_t st);
 
 // Tensor-core GEMM launchers (k_tc_*.cu), one per fused epilogue.
+int qkv_split_for(const Model& m);
+cudaError_t tc_gemm_part(int nb, const CUtensorMap& x, const TcParams& p, cudaStream_t st);
 cudaError_t tc_gemm_qkv(int nb, const CUtensorMap& x, const TcParams& p,
                         cudaStream_t st);
 cudaError_t tc_gemm_resid(int nb, const CUtensorMap& x, const TcParams& p,

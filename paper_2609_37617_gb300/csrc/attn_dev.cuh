@@ -60,14 +60,102 @@ struct AttnArgs {
   int parts_max, qmax;
   bf16* ao;             // [2 rows][nq * D]: hi rows, then lo rows from lo_row
   int lo_row;
+  // split-K sums of the QKV projection (TC_PART), when attention finishes them
+  const float* qkv_part;  // [tile][split][qkv_ld][128], tile = column / 128
+  const float* qkv_rinv;  // [qkv_ld] 1 / rms of each token row
+  const float2* rope;     // [rows][D / 2] (cos, sin)
+  int qkv_split, qkv_ld;
 };
 
+// ---- finishing the QKV projection from its split-K sums ----------------------
+
+// Projection value of column col (q, k or v head * D + e) for token row gm:
+// the split parts added in rank order, times the row's 1 / rms.
+__device__ __forceinline__ float qkv_value(const AttnArgs& a, int col, int gm) {
+  const float* src = a.qkv_part + ((size_t)(col >> 7) * a.qkv_split * a.qkv_ld + gm) * 128 + (col & 127);
+  float v[8];
+#pragma unroll
+  for (int r = 0; r < 8; ++r) v[r] = r < a.qkv_split ? src[(size_t)r * a.qkv_ld * 128] : 0.f;
+  float acc = 0.f;
+#pragma unroll
+  for (int r = 0; r < 8; ++r)
+    if (r < a.qkv_split) acc += v[r];
+  return acc * a.qkv_rinv[gm];
+}
+
+// Rotate-half RoPE of the pair (x at e, xp at e + D/2): returns the rotated
+// value at e (first) and at e + D/2 (second).
+__device__ __forceinline__ float2 rope_pair(float x, float xp, float2 cs) {
+  return make_float2(fmaf(x, cs.x, -(xp * cs.y)), fmaf(xp, cs.x, x * cs.y));
+}
+
+// Rotated query / key pair (e, e + D/2) of head `head` (column head * D) at
+// token row gm, e < D/2.
+template <int D>
+__device__ __forceinline__ float2 qk_rotated(const AttnArgs& a, int head, int e, int gm) {
+  const float x = qkv_value(a, head * D + e, gm), xp = qkv_value(a, head * D + e + D / 2, gm);
+  return rope_pair(x, xp, a.rope[(size_t)gm * (D / 2) + e]);
+}
+
+
+// Stages keys/values [p0, p0 + 64) of the item into sK/sV: rows below `from`
+// are left alone, rows in [from, kend) are copied from the cache (cp.async,
+// committed), rows at or beyond kend are zero.
+template <int D>
+__device__ __forceinline__ void stage_kv(const AttnArgs& a, int layer, int part, int g, int b,
+                                         int from, bf16 (*sK)[kPitch], bf16 (*sV)[kPitch],
+                                         int tid, int nthr, int upto) {
+  const int p0 = part * kPart;
+  const size_t head = (((size_t)layer * a.batch + b) * a.nkv + g) * (size_t)a.cap;
+  constexpr int SEGS = D / 8;  // 16-byte pieces per row
+  for (int idx = tid; idx < kPart * SEGS; idx += nthr) {
+    const int t = idx / SEGS, sg = idx - t * SEGS;
+    const int pos = p0 + t;
+    if (pos < from) continue;
+    if (pos < upto) {
+      cp_async16(&sK[t][sg * 8], a.kc + (head + pos) * D + sg * 8);
+      cp_async16(&sV[t][sg * 8], a.vc + (head + pos) * D + sg * 8);
+    } else {
+      *reinterpret_cast<uint4*>(&sK[t][sg * 8]) = make_uint4(0, 0, 0, 0);
+      *reinterpret_cast<uint4*>(&sV[t][sg * 8]) = make_uint4(0, 0, 0, 0);
+    }
+  }
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+
+// The item's keys/values already in the cache ([0, L) of the request) go to
+// sK/sV before the block's own rows exist (cp.async, committed); positions at
+// or beyond L + M are zero.  Rows [L, L + M) are left for part_item.
+template <int D>
+__device__ __forceinline__ void stage_old_kv(const AttnArgs& a, int layer, int part, int g,
+                                             int b, bf16 (*sK)[kPitch], bf16 (*sV)[kPitch],
+                                             int tid, int nthr) {
+  const int L = a.len[b], M = a.rm.start[b + 1] - a.rm.start[b];
+  const int p0 = part * kPart;
+  if (p0 >= L + M) return;
+  const size_t head = (((size_t)layer * a.batch + b) * a.nkv + g) * (size_t)a.cap;
+  constexpr int SEGS = D / 8;
+  for (int idx = tid; idx < kPart * SEGS; idx += nthr) {
+    const int t = idx / SEGS, sg = idx - t * SEGS;
+    const int pos = p0 + t;
+    if (pos < L) {
+      cp_async16(&sK[t][sg * 8], a.kc + (head + pos) * D + sg * 8);
+      cp_async16(&sV[t][sg * 8], a.vc + (head + pos) * D + sg * 8);
+    } else if (pos >= L + M) {
+      *reinterpret_cast<uint4*>(&sK[t][sg * 8]) = make_uint4(0, 0, 0, 0);
+      *reinterpret_cast<uint4*>(&sV[t][sg * 8]) = make_uint4(0, 0, 0, 0);
+    }
+  }
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
 
 // Split-KV item: keys [64 part, 64 part + 64) of kv head g of request b for
 // all (k + 1) * group queries; writes the partition's (max, sum) and
 // unnormalised output per query.  nthr threads (a multiple of 32) of the
 // calling group, thread index tid, barrier bar_id; sK/sV hold 64 x kPitch bf16.
-template <int D>
+// OLD_STAGED: rows [0, L) (and zeros at or beyond L + M) were staged by
+// stage_old_kv; only the block's own rows [L, L + M) are copied here.
+template <int D, bool OLD_STAGED = false>
 __device__ __forceinline__ void part_item(const AttnArgs& a, int layer, int part, int g, int b,
                                           bf16 (*sK)[kPitch], bf16 (*sV)[kPitch], int tid,
                                           int nthr, int bar_id) {
@@ -79,22 +167,7 @@ __device__ __forceinline__ void part_item(const AttnArgs& a, int layer, int part
   if (p0 >= kend) return;  // uniform over the CTA
   const int Qn = M * G;
 
-
-  // stage keys/values [p0, p0 + 64); rows at or beyond kend are zero
-  const size_t head = (((size_t)layer * a.batch + b) * a.nkv + g) * (size_t)a.cap;
-  constexpr int SEGS = D / 8;  // 16-byte pieces per row
-  for (int idx = tid; idx < kPart * SEGS; idx += nthr) {
-    const int t = idx / SEGS, sg = idx - t * SEGS;
-    const int pos = p0 + t;
-    if (pos < kend) {
-      cp_async16(&sK[t][sg * 8], a.kc + (head + pos) * D + sg * 8);
-      cp_async16(&sV[t][sg * 8], a.vc + (head + pos) * D + sg * 8);
-    } else {
-      *reinterpret_cast<uint4*>(&sK[t][sg * 8]) = make_uint4(0, 0, 0, 0);
-      *reinterpret_cast<uint4*>(&sV[t][sg * 8]) = make_uint4(0, 0, 0, 0);
-    }
-  }
-  asm volatile("cp.async.commit_group;" ::: "memory");
+  stage_kv<D>(a, layer, part, g, b, OLD_STAGED ? L : 0, sK, sV, tid, nthr, kend);
 
   const int warp = tid >> 5, lane = tid & 31;
   const int gq = lane >> 2, tq = lane & 3;

@@ -27,8 +27,13 @@
 //     count per tile) adds the parts in CTA order and applies the epilogue:
 //     the sum order depends on (N, K, grid) only, never on the number of
 //     token rows or on arrival order, so results are batch invariant;
-//   * the epilogue is fused: RoPE + KV-cache append (QKV), residual add
-//     (O, down), SwiGLU (gate/up), and logits + argmax (LM head).
+//   * the epilogue is fused: residual add (O, down), SwiGLU (gate/up), and
+//     logits + argmax (LM head).  The QKV projection (TC_PART) instead splits
+//     K evenly over a fixed number of CTAs per tile and stores each CTA's
+//     unscaled sums: the attention's first kernel adds them, applies RoPE and
+//     appends the keys and values, so no CTA of this kernel waits for
+//     another's part at its end.  (TC_QKV, the same epilogue done here by the
+//     last CTA of a tile, serves the persistent whole-pass kernel.)
 // Every mbarrier wait is bounded in time; on expiry the kernel records an
 // error bit, drains its own outstanding copies and MMAs, frees TMEM and exits.
 #pragma once
@@ -71,6 +76,22 @@ __device__ __forceinline__ unsigned long long tc_pack_best(float v, int idx) {
   uint32_t u = __float_as_uint(v);
   uint32_t key = (u & 0x80000000u) ? ~u : (u | 0x80000000u);
   return ((unsigned long long)key << 32) | (unsigned long long)(0xFFFFFFFFu - (uint32_t)idx);
+}
+
+// TC_PART: CTA c takes k-blocks [r kb / split, (r + 1) kb / split) of tile
+// c / split (r = c mod split); otherwise the stream-K range of tc_start.
+// Either way the decomposition depends on (N, K, the device) only, never on
+// the number of token rows.
+__device__ __forceinline__ long long tc_start(int c, const TcParams& p);
+__device__ __forceinline__ void tc_range(int c, const TcParams& p, long long& u0, long long& u1) {
+  if (p.split > 1) {
+    const int tile = c / p.split, r = c - tile * p.split;
+    u0 = (long long)tile * p.kb + (long long)r * p.kb / p.split;
+    u1 = (long long)tile * p.kb + (long long)(r + 1) * p.kb / p.split;
+  } else {
+    u0 = tc_start(c, p);
+    u1 = tc_start(c + 1, p);
+  }
 }
 
 __device__ __forceinline__ long long tc_start(int c, const TcParams& p) {
@@ -286,6 +307,8 @@ __device__ __forceinline__ void tc_row_prologue(const TcParams& p, float* s_rinv
           for (int u = 0; u < 32; ++u) tot += v[u];
         }
         s_rinv[m] = rsqrtf(tot / (float)p.hidden + p.eps);
+        // TC_PART leaves the scaling to the kernel that finishes its sums
+        if (EPI == TC_PART && blockIdx.x == 0) p.part_rinv[gm] = s_rinv[m];
       }
       if (EPI == TC_QKV) {
         s_req[m] = b;
@@ -392,7 +415,8 @@ __global__ void __launch_bounds__(192, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int c = blockIdx.x;
-  const long long u0 = tc_start(c, p), u1 = tc_start(c + 1, p);
+  long long u0, u1;
+  tc_range(c, p, u0, u1);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
@@ -542,7 +566,20 @@ __global__ void __launch_bounds__(192, 1)
       }
       ptx::tc_fence_after();
       const uint32_t tbase = tmem + (uint32_t)(buf * ACC_COLS) + ((uint32_t)(q4 * 32) << 16);
-      if (whole) {
+      if (EPI == TC_PART) {
+        // this CTA's k-block sums for its tile, unscaled, [row][tile row]
+        float* dst = p.part + ((size_t)c * p.part_ld + p.row0) * 128 + nl;
+        for (int ch = 0; ch < nchunks; ++ch) {
+          uint32_t v[16];
+          tc_load_acc<NB>(tbase, ch, v);
+#pragma unroll
+          for (int j = 0; j < CH; ++j)
+            if (ch * CH + j < p.rows) dst[(size_t)(ch * CH + j) * 128] = __uint_as_float(v[j]);
+        }
+        ptx::tc_fence_before();
+        __syncwarp();
+        if (lane == 0) ptx::mbar_arrive(&acc_empty[buf]);
+      } else if (whole) {
         for (int ch = 0; ch < nchunks; ++ch) {
           uint32_t v[16];
           tc_load_acc<NB>(tbase, ch, v);

@@ -8,8 +8,14 @@
 // head, for all k + 1 rows, form one query matrix of (k + 1) * G rows, so each
 // key/value entry is read from HBM once per block.
 //
+// Pass 0 (qkv_finish_kernel): the QKV projection arrives as split-K partial
+// sums (TC_PART); one CTA per (token row, head) adds them in rank order,
+// scales by the row's 1 / rms, rotates (RoPE) and writes the queries, and
+// appends the new keys and values to the cache.
 // Pass 1 (attn_part_kernel): one CTA per (64-key partition, kv head, request).
-// Keys and values are staged in shared memory; each warp takes 16 query rows;
+// Keys and values are staged in shared memory -- those already in the cache
+// before the kernel waits for pass 0, the block's own after; each warp takes
+// 16 query rows;
 // S = Q K^T and O = P V run on the tensor cores (mma.sync m16n8k16, bf16 in,
 // fp32 accumulate), with Q and P each split into bf16 hi + lo parts (two MMAs)
 // so that only the bf16 cache itself limits precision; the softmax runs in
@@ -27,11 +33,43 @@ using namespace attn;
 
 template <int D>
 __global__ void __launch_bounds__(256, 1) attn_part_kernel(AttnArgs a) {
-  ptx::griddep_wait();
-  ptx::griddep_launch_dependents();
   __shared__ __align__(16) bf16 sK[kPart][kPitch];
   __shared__ __align__(16) bf16 sV[kPart][kPitch];
-  part_item<D>(a, a.layer, blockIdx.x, blockIdx.y, blockIdx.z, sK, sV, threadIdx.x, blockDim.x, 0);
+  // the keys/values already in the cache do not depend on the predecessor
+  stage_old_kv<D>(a, a.layer, blockIdx.x, blockIdx.y, blockIdx.z, sK, sV, threadIdx.x, blockDim.x);
+  ptx::griddep_wait();
+  ptx::griddep_launch_dependents();
+  part_item<D, true>(a, a.layer, blockIdx.x, blockIdx.y, blockIdx.z, sK, sV, threadIdx.x,
+                     blockDim.x, 0);
+}
+
+// The QKV projection finished from its split-K sums (TC_PART): one CTA of
+// D / 2 threads per (token row, head); thread e
+// forms the pair (e, e + D/2) -- rotated queries into q, rotated keys and
+// values appended to the cache.  Every load of a thread is issued before the
+// first is used.
+template <int D>
+__global__ void __launch_bounds__(D / 2) qkv_finish_kernel(AttnArgs a) {
+  ptx::griddep_wait();
+  ptx::griddep_launch_dependents();
+  constexpr int H2 = D / 2;
+  const int gm = blockIdx.x, head = blockIdx.y, e = threadIdx.x;
+  const int b = row_request(a.rm, gm), pos = a.len[b] + (gm - a.rm.start[b]);
+  const float2 y = (head < a.nq + a.nkv) ? qk_rotated<D>(a, head, e, gm)
+                                         : make_float2(qkv_value(a, head * D + e, gm),
+                                                       qkv_value(a, head * D + e + H2, gm));
+  if (head < a.nq) {
+    float* q = const_cast<float*>(a.q) + (size_t)gm * a.nq * D + head * D;
+    q[e] = y.x;
+    q[e + H2] = y.y;
+  } else {
+    const bool is_k = head < a.nq + a.nkv;
+    const int g = is_k ? head - a.nq : head - a.nq - a.nkv;
+    bf16* dst = const_cast<bf16*>(is_k ? a.kc : a.vc) +
+                ((((size_t)a.layer * a.batch + b) * a.nkv + g) * a.cap + pos) * D;
+    dst[e] = __float2bfloat16_rn(y.x);
+    dst[e + H2] = __float2bfloat16_rn(y.y);
+  }
 }
 
 template <int D>
@@ -76,13 +114,21 @@ cudaError_t launch_attention_split(const RowMap& m, const Model& md, KvState& kv
   const int parts = (int)((max_len + kPart - 1) / kPart);
   dim3 g1(parts, c.n_kv_heads, kv.batch);
   dim3 g2(m.rows, c.n_q_heads);
+  a.qkv_part = kv.qkv_part;
+  a.qkv_rinv = kv.qkv_rinv;
+  a.rope = kv.rope;
+  a.qkv_split = kv.qkv_split;
+  a.qkv_ld = kv.rows_alloc;
+  const dim3 gf(m.rows, c.n_q_heads + 2 * c.n_kv_heads);
   cudaError_t e;
-  kv.launches += 2;
+  kv.launches += 3;
   if (c.head_dim == 128) {
-    e = launch_pdl(attn_part_kernel<128>, g1, dim3(256), 0, st, a);
+    e = launch_pdl(qkv_finish_kernel<128>, gf, dim3(64), 0, st, a);
+    if (e == cudaSuccess) e = launch_pdl(attn_part_kernel<128>, g1, dim3(256), 0, st, a);
     if (e == cudaSuccess) e = launch_pdl(attn_merge_kernel<128>, g2, dim3(128), 0, st, a);
   } else {
-    e = launch_pdl(attn_part_kernel<64>, g1, dim3(256), 0, st, a);
+    e = launch_pdl(qkv_finish_kernel<64>, gf, dim3(32), 0, st, a);
+    if (e == cudaSuccess) e = launch_pdl(attn_part_kernel<64>, g1, dim3(256), 0, st, a);
     if (e == cudaSuccess) e = launch_pdl(attn_merge_kernel<64>, g2, dim3(64), 0, st, a);
   }
   return e;

@@ -9,6 +9,7 @@
 namespace as2d {
 namespace ptx {
 
+
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return (uint32_t)__cvta_generic_to_shared(p);
 }
