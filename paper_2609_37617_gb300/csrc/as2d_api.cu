@@ -395,8 +395,24 @@ cudaError_t tc_project(int epi, const Model& m, KvState& s, const RowMap& rm, co
   p.n_tiles = (N + 127) / 128;
   p.kb = (K + 63) / 64;
   p.units = (long long)p.n_tiles * p.kb;
+  // Work split (all of it a function of N, K and the device only, so a
+  // row's sums are added in the same order whatever the number of rows):
+  //   QKV (TC_PART): K split evenly over qkv_split CTAs per tile, sums
+  //     finished by qkv_finish_kernel;
+  //   at least as many tiles as SMs (gate/up): whole tiles per CTA, as
+  //     evenly as they go, each finished by its own CTA;
+  //   otherwise stream-K over one CTA per SM; residual projections leave
+  //     their split tiles to tc_reduce_kernel, the LM head finishes them in
+  //     the GEMM (last CTA of a tile).
   p.grid = (int)(p.units < m.sm_count ? p.units : m.sm_count);
   p.split = 0;
+  p.defer = epi == TC_RESID ? 1 : 0;
+  if (epi == TC_SWIGLU && p.n_tiles >= m.sm_count) {
+    const int per = (p.n_tiles + m.sm_count - 1) / m.sm_count;
+    p.split = 1;
+    p.grid = (p.n_tiles + per - 1) / per;
+    p.defer = 0;
+  }
   if (epi == TC_PART) {
     p.split = s.qkv_split;
     p.grid = p.n_tiles * p.split;
@@ -423,7 +439,7 @@ cudaError_t tc_project(int epi, const Model& m, KvState& s, const RowMap& rm, co
       default: e = tc_gemm_logits(nb, x, p, st); break;
     }
     if (e != cudaSuccess) return e;
-    s.launches += 1;
+    s.launches += (p.defer && p.grid >= 2) ? 2 : 1;
   }
   return cudaSuccess;
 }

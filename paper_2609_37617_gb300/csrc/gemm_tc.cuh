@@ -88,6 +88,10 @@ __device__ __forceinline__ void tc_range(int c, const TcParams& p, long long& u0
     const int tile = c / p.split, r = c - tile * p.split;
     u0 = (long long)tile * p.kb + (long long)r * p.kb / p.split;
     u1 = (long long)tile * p.kb + (long long)(r + 1) * p.kb / p.split;
+  } else if (p.split == 1) {
+    // whole tiles [c T / grid, (c + 1) T / grid)
+    u0 = ((long long)c * p.n_tiles / p.grid) * p.kb;
+    u1 = ((long long)(c + 1) * p.n_tiles / p.grid) * p.kb;
   } else {
     u0 = tc_start(c, p);
     u1 = tc_start(c + 1, p);
@@ -610,6 +614,10 @@ __global__ void __launch_bounds__(192, 1)
         ptx::tc_fence_before();
         __syncwarp();
         if (lane == 0) ptx::mbar_arrive(&acc_empty[buf]);
+        if (p.defer) {  // finished by tc_reduce_kernel, launched next
+          u = send;
+          continue;
+        }
         // the last CTA to store a part of this tile adds the parts, in CTA
         // order whichever CTA that is, and applies the epilogue
         __threadfence();
@@ -638,6 +646,27 @@ __global__ void __launch_bounds__(192, 1)
   }
 }
 
+// Finishes the tiles a stream-K launch left split between CTAs (p.defer):
+// one CTA of 128 threads per tile; the parts, the epilogue's operands and
+// the row prologue's loads are issued together (tc_reduce_tile).
+template <int NB, int EPI>
+__global__ void __launch_bounds__(128) tc_reduce_kernel(const __grid_constant__ TcParams p) {
+  using Sh = TcShape<NB>;
+  constexpr int SP = Sh::SP;
+  __shared__ float sC[128 * SP];
+  __shared__ float s_rinv[NB];
+  __shared__ float red[64];
+  __shared__ int s_pos[NB], s_req[NB];
+  const int tile = blockIdx.x;
+  const long long tstart = (long long)tile * p.kb, tend = tstart + p.kb;
+  const int c_first = tc_owner(tstart, p), c_last = tc_owner(tend - 1, p);
+  ptx::griddep_wait();
+  ptx::griddep_launch_dependents();
+  if (c_last == c_first) return;  // a whole tile, finished by its GEMM CTA
+  tc_reduce_tile<NB, EPI, 8, true>(p, sC, s_rinv, red, s_pos, s_req, tile, c_first,
+                                   c_last - c_first + 1, threadIdx.x, threadIdx.x);
+}
+
 template <int NB, int EPI>
 cudaError_t tc_gemm_launch(const CUtensorMap& x, const TcParams& p, cudaStream_t st) {
   constexpr uint32_t smem = TcShape<NB>::SMEM;
@@ -648,7 +677,9 @@ cudaError_t tc_gemm_launch(const CUtensorMap& x, const TcParams& p, cudaStream_t
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  return launch_pdl(tc_gemm_kernel<NB, EPI>, dim3(p.grid), dim3(192), smem, st, x, p);
+  cudaError_t e = launch_pdl(tc_gemm_kernel<NB, EPI>, dim3(p.grid), dim3(192), smem, st, x, p);
+  if (e != cudaSuccess || !p.defer || p.grid < 2) return e;
+  return launch_pdl(tc_reduce_kernel<NB, EPI>, dim3(p.n_tiles), dim3(128), 0, st, p);
 }
 
 template <int EPI>
