@@ -667,6 +667,54 @@ __global__ void __launch_bounds__(128) tc_reduce_kernel(const __grid_constant__ 
                                    c_last - c_first + 1, threadIdx.x, threadIdx.x);
 }
 
+// The residual epilogue of a stream-K launch's split tiles, one CTA of 128
+// threads per (tile, token row): thread n adds the parts of tile row n in CTA
+// order, adds the residual, writes h and the next operand (hi, lo) and takes
+// its share of the row's sum of squares -- the arithmetic of
+// tc_reduce_tile + TC_RESID, with every load of a thread issued first.
+template <int NB>
+__global__ void __launch_bounds__(128) tc_resid_finish_kernel(const __grid_constant__ TcParams p) {
+  __shared__ float red[4];
+  const int tile = blockIdx.x, m = blockIdx.y, n = threadIdx.x;
+  const long long tstart = (long long)tile * p.kb, tend = tstart + p.kb;
+  const int c_first = tc_owner(tstart, p), c_last = tc_owner(tend - 1, p);
+  ptx::griddep_wait();
+  ptx::griddep_launch_dependents();
+  if (c_last == c_first) return;  // a whole tile, finished by its GEMM CTA
+  const int nparts = c_last - c_first + 1;
+  const int col = tile * 128 + n;
+  const size_t at = (size_t)(p.row0 + m) * p.N + col;
+  const float h0 = p.h[at], gn = p.g_next[col];
+  float acc = 0.f;
+  for (int part0 = 0; part0 < nparts; part0 += 8) {
+    float v[8];
+#pragma unroll
+    for (int pp = 0; pp < 8; ++pp) {
+      v[pp] = 0.f;
+      if (part0 + pp < nparts) {
+        const int cp = c_first + part0 + pp;
+        const int sl = (cp == c_first && (int)(tc_start(cp, p) / p.kb) != tile) ? 1 : 0;
+        v[pp] = __ldcg(p.ws + ((size_t)(cp * 2 + sl) * 128 + n) * NB + m);
+      }
+    }
+#pragma unroll
+    for (int pp = 0; pp < 8; ++pp)
+      if (part0 + pp < nparts) acc += v[pp];
+  }
+  const float hn = h0 + acc;
+  p.h[at] = hn;
+  const float xv = hn * gn;
+  const bf16 xh = __float2bfloat16_rn(xv);
+  p.xn[at] = xh;
+  p.xn[at + (size_t)p.lo_row * p.N] = __float2bfloat16_rn(xv - __bfloat162float(xh));
+  float sq = hn * hn;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xFFFFFFFFu, sq, o);
+  if ((n & 31) == 0) red[n >> 5] = sq;
+  __syncthreads();
+  if (n == 0) p.ss[(size_t)tile * p.ss_ld + p.row0 + m] = ((red[0] + red[1]) + red[2]) + red[3];
+}
+
 template <int NB, int EPI>
 cudaError_t tc_gemm_launch(const CUtensorMap& x, const TcParams& p, cudaStream_t st) {
   constexpr uint32_t smem = TcShape<NB>::SMEM;
@@ -679,6 +727,8 @@ cudaError_t tc_gemm_launch(const CUtensorMap& x, const TcParams& p, cudaStream_t
   }
   cudaError_t e = launch_pdl(tc_gemm_kernel<NB, EPI>, dim3(p.grid), dim3(192), smem, st, x, p);
   if (e != cudaSuccess || !p.defer || p.grid < 2) return e;
+  if (EPI == TC_RESID)
+    return launch_pdl(tc_resid_finish_kernel<NB>, dim3(p.n_tiles, p.rows), dim3(128), 0, st, p);
   return launch_pdl(tc_reduce_kernel<NB, EPI>, dim3(p.n_tiles), dim3(128), 0, st, p);
 }
 
