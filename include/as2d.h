@@ -47,6 +47,7 @@ typedef int32_t as2d_status;
 #define AS2D_ERR_CUDA (-3)          /* a CUDA runtime call failed            */
 #define AS2D_ERR_UNSUPPORTED (-4)   /* shape outside what the kernels handle */
 #define AS2D_ERR_DEVICE (-5)        /* a kernel reported an error or timeout */
+#define AS2D_ERR_NO_MEMORY (-6)     /* a host allocation failed              */
 
 /* Largest number of candidates per request in one call (the budget b of
    App. A.2; physical width K = k + 1 <= 17). */
@@ -227,6 +228,99 @@ as2d_status as2d_kv_profile_read(as2d_kv* kv, int32_t* launches,
 
 void as2d_kv_free(as2d_kv* kv);
 void as2d_model_free(as2d_model* model);
+
+/* ---- Candidate buffer, read cursor and alignment -------------------------
+   (Section 3.1 "Ordered publication and buffering"; Section 3.2 "Candidate
+   alignment"; App. B.1 "Source records and incremental publication"; App. B.3
+   "Candidate alignment"; Fig. 4.)  Host-side: one buffer per request and
+   source.  The producer appends immutable batches of at most
+   AS2D_CBUF_BATCH tokens; verification reads a snapshot of what is published
+   from a read cursor that only alignment moves.  Alignment changes the
+   cursor, never published tokens, committed tokens or the target's state, so
+   the committed text is the target's greedy text whatever the buffer holds
+   (Prop. 1).  Every entry point below is safe to call from several host
+   threads at once (a producer thread publishing while the verifier reads):
+   each one is atomic with respect to the others on the same buffer.
+
+   Alignment, after a call that verified k candidates from cursor c,
+   accepted n of them and ended with the target's token x (the correction,
+   or the bonus token when n == k), with search bound W (the window):
+     R1  x stands at buffer position m = c + n.  Once the buffer holds x at m
+         (possible only after full acceptance; re-checked at each
+         as2d_cbuf_candidates until m is published), the cursor steps over it
+         to m + 1.
+     R2  Otherwise m stays eligible: the next call verifies root x followed by
+         the candidates from m (x may be a target insertion); if it accepts
+         n >= 1, R1 applies to it.
+     R3  If it accepts none, its token t is the first alignment anchor: the
+         cursor moves to j + 1 for the first j in (m, m + W] holding t, else
+         to j + 2 for the first j in [m, m + W] holding x, else the target
+         decodes alone (k = 0).  While it does, its latest token is looked for
+         before each call in the published positions [s, s + W), s starting
+         at m + 1 and growing by one per token decoded alone; a match at j
+         moves the cursor to j + 1. */
+#define AS2D_CBUF_BATCH 8
+#define AS2D_CBUF_NORMAL 0   /* candidates follow the cursor              */
+#define AS2D_CBUF_REALIGN 1  /* R1/R2: waiting on the token at m          */
+#define AS2D_CBUF_ALONE 2    /* R3: no usable candidates; k = 0           */
+
+/* Source record of one published batch (App. B.1).  confidence is
+   meaningful only when has_confidence != 0. */
+typedef struct as2d_source_record {
+  int32_t request, source, producer, offset;
+  double time;
+  float confidence;
+  int32_t has_confidence;
+} as2d_source_record;
+
+typedef struct as2d_cbuf as2d_cbuf;
+
+/* Create an empty buffer with search bound `window` in [1, 1024]. */
+as2d_status as2d_cbuf_create(int32_t window, as2d_cbuf** out);
+
+/* Append one batch: tokens host int32 [n], 1 <= n <= AS2D_CBUF_BATCH, every
+   id >= 0; rec (host, required) is copied.  Published tokens never change. */
+as2d_status as2d_cbuf_publish(as2d_cbuf* buf, const int32_t* tokens, int32_t n,
+                              const as2d_source_record* rec);
+
+/* The candidates for the next verification call: applies the checks that
+   wait on publication (R1's step-over, R3's search while decoding alone),
+   then copies up to b (0 <= b <= AS2D_MAX_K) published tokens from the cursor
+   into host int32 tokens[b] and their number into *k (0 while the target
+   decodes alone).  The next as2d_cbuf_after_call must report that k. */
+as2d_status as2d_cbuf_candidates(as2d_cbuf* buf, int32_t b, int32_t* tokens,
+                                 int32_t* k);
+
+/* Report the call's outcome: the k of the last as2d_cbuf_candidates,
+   n_accepted in [0, k] and the call's final token (correction or bonus,
+   >= 0).  Moves the cursor by R1-R3. */
+as2d_status as2d_cbuf_after_call(as2d_cbuf* buf, int32_t k, int32_t n_accepted,
+                                 int32_t correction);
+
+/* Published token count, cursor and mode (AS2D_CBUF_*); any may be NULL. */
+as2d_status as2d_cbuf_state(as2d_cbuf* buf, int32_t* ready, int32_t* cursor,
+                            int32_t* mode);
+
+/* Copy the source record of the batch that published `position`
+   (AS2D_ERR_INVALID_ARG if the position is not published). */
+as2d_status as2d_cbuf_source_of(as2d_cbuf* buf, int32_t position,
+                                as2d_source_record* out);
+
+void as2d_cbuf_free(as2d_cbuf* buf);
+
+/* One verification call driven by candidate buffers: bufs is a host array of
+   kv's batch buffers (request r reads bufs[r]).  Takes up to b candidates
+   from each buffer, copies them to the device, runs as2d_verify_block on
+   `stream`, reads n_accepted and the correction back (this synchronises the
+   stream) and reports them to each buffer.  Outputs (host, may be NULL):
+   k_used int32 [batch]; committed int32 [batch][b + 1], row r holding the
+   request's n_r + 1 committed tokens (accepted candidates, then the
+   correction); n_committed int32 [batch] = n_r + 1.  Device staging memory
+   is allocated on the first call and kept until as2d_kv_free.  Errors of
+   as2d_verify_block are returned as they are, before any buffer changes. */
+as2d_status as2d_verify_from_buffers(as2d_kv* kv, as2d_cbuf* const* bufs, int32_t b,
+                                     int32_t* k_used, int32_t* committed,
+                                     int32_t* n_committed, void* stream);
 
 /* Thread-local description of the last error ("" if none). */
 const char* as2d_last_error(void);

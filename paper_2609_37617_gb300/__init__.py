@@ -25,6 +25,9 @@ AS2D_ERR_CAPACITY = -2
 AS2D_ERR_CUDA = -3
 AS2D_ERR_UNSUPPORTED = -4
 AS2D_ERR_DEVICE = -5
+AS2D_ERR_NO_MEMORY = -6
+AS2D_CBUF_BATCH = 8
+CBUF_MODES = {0: "normal", 1: "realign", 2: "alone"}
 AS2D_MAX_K = 16
 AS2D_MAX_BATCH = 64
 
@@ -32,7 +35,10 @@ EXPORTED = ("as2d_model_load", "as2d_kv_init_prefilled", "as2d_verify_block",
             "as2d_decode_step", "as2d_kv_rollback", "as2d_kv_read_state",
             "as2d_kv_device_state", "as2d_kv_check", "as2d_kv_free",
             "as2d_model_free", "as2d_last_error", "as2d_kv_profile",
-            "as2d_kv_profile_read", "as2d_decode_step_static")
+            "as2d_kv_profile_read", "as2d_decode_step_static", "as2d_cbuf_create",
+            "as2d_cbuf_publish", "as2d_cbuf_candidates", "as2d_cbuf_after_call",
+            "as2d_cbuf_state", "as2d_cbuf_source_of", "as2d_cbuf_free",
+            "as2d_verify_from_buffers")
 KERNEL_CLASSES = {"qkv": 0, "attention": 1, "o": 2, "gate_up": 3, "down": 4,
                   "lm_head": 5, "other": 6, "pass": 7}
 
@@ -54,6 +60,13 @@ class as2d_weights(ctypes.Structure):
 class as2d_verify_out(ctypes.Structure):
     _fields_ = [("n_accepted", ctypes.c_void_p), ("correction_token", ctypes.c_void_p),
                 ("greedy", ctypes.c_void_p), ("logits", ctypes.c_void_p)]
+
+
+class as2d_source_record(ctypes.Structure):
+    _fields_ = [("request", ctypes.c_int32), ("source", ctypes.c_int32),
+                ("producer", ctypes.c_int32), ("offset", ctypes.c_int32),
+                ("time", ctypes.c_double), ("confidence", ctypes.c_float),
+                ("has_confidence", ctypes.c_int32)]
 
 
 _P = ctypes.c_void_p
@@ -89,6 +102,19 @@ _lib.as2d_kv_profile_read.argtypes = [_P, ctypes.POINTER(ctypes.c_int32),
 _lib.as2d_kv_profile_read.restype = _S
 _lib.as2d_decode_step_static.argtypes = [_P, _P, _P, ctypes.c_int32, _P, _P, _P, _P, _P]
 _lib.as2d_decode_step_static.restype = _S
+_lib.as2d_cbuf_create.argtypes = [_S, ctypes.POINTER(ctypes.c_void_p)]
+_lib.as2d_cbuf_publish.argtypes = [_P, _P, _S, ctypes.POINTER(as2d_source_record)]
+_lib.as2d_cbuf_candidates.argtypes = [_P, _S, _P, ctypes.POINTER(ctypes.c_int32)]
+_lib.as2d_cbuf_after_call.argtypes = [_P, _S, _S, _S]
+_lib.as2d_cbuf_state.argtypes = [_P, _P, _P, _P]
+_lib.as2d_cbuf_source_of.argtypes = [_P, _S, ctypes.POINTER(as2d_source_record)]
+_lib.as2d_cbuf_free.argtypes = [_P]
+_lib.as2d_cbuf_free.restype = None
+_lib.as2d_verify_from_buffers.argtypes = [_P, _P, _S, _P, _P, _P, _P]
+for _n in ("as2d_cbuf_create", "as2d_cbuf_publish", "as2d_cbuf_candidates",
+           "as2d_cbuf_after_call", "as2d_cbuf_state", "as2d_cbuf_source_of",
+           "as2d_verify_from_buffers"):
+    getattr(_lib, _n).restype = _S
 _lib.as2d_last_error.argtypes = []
 _lib.as2d_last_error.restype = ctypes.c_char_p
 
@@ -212,6 +238,56 @@ def as2d_decode_step_static(model, k_cache_ptr, v_cache_ptr, capacity, len_ptr, 
                                         _P(int(stream) or None))
 
 
+def as2d_cbuf_create(window):
+    h = ctypes.c_void_p()
+    st = _lib.as2d_cbuf_create(window, ctypes.byref(h))
+    return st, h.value
+
+
+def as2d_cbuf_publish(buf, tokens, record):
+    arr = _i32_array(tokens) if len(tokens) else None
+    return _lib.as2d_cbuf_publish(buf, arr, len(tokens),
+                                  ctypes.byref(record) if record is not None else None)
+
+
+def as2d_cbuf_candidates(buf, b):
+    arr = (ctypes.c_int32 * max(b, 1))()
+    k = ctypes.c_int32(-1)
+    st = _lib.as2d_cbuf_candidates(buf, b, arr, ctypes.byref(k))
+    return st, list(arr[:max(k.value, 0)])
+
+
+def as2d_cbuf_after_call(buf, k, n_accepted, correction):
+    return _lib.as2d_cbuf_after_call(buf, k, n_accepted, correction)
+
+
+def as2d_cbuf_state(buf):
+    r, c, m = ctypes.c_int32(), ctypes.c_int32(), ctypes.c_int32()
+    st = _lib.as2d_cbuf_state(buf, ctypes.byref(r), ctypes.byref(c), ctypes.byref(m))
+    return st, r.value, c.value, m.value
+
+
+def as2d_cbuf_source_of(buf, position):
+    rec = as2d_source_record()
+    st = _lib.as2d_cbuf_source_of(buf, position, ctypes.byref(rec))
+    return st, rec
+
+
+def as2d_cbuf_free(buf):
+    _lib.as2d_cbuf_free(buf)
+
+
+def as2d_verify_from_buffers(kv, bufs, b, batch, stream=0):
+    """Returns (status, k_used, committed lists)."""
+    hb = (ctypes.c_void_p * batch)(*bufs)
+    k_used = (ctypes.c_int32 * batch)()
+    comm = (ctypes.c_int32 * (batch * (b + 1)))()
+    ncomm = (ctypes.c_int32 * batch)()
+    st = _lib.as2d_verify_from_buffers(kv, hb, b, k_used, comm, ncomm, stream)
+    rows = [list(comm[r * (b + 1): r * (b + 1) + ncomm[r]]) for r in range(batch)]
+    return st, list(k_used), rows
+
+
 def exported_symbols():
     """Names of include/as2d.h's entry points that the loaded library exports."""
     return [n for n in EXPORTED if hasattr(_lib, n)]
@@ -236,6 +312,55 @@ class Model:
     def close(self):
         if self.handle:
             as2d_model_free(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+class CandidateBuffer:
+    """Owns an as2d_cbuf: one request's published candidates, read cursor and
+    alignment state (host side)."""
+
+    def __init__(self, window=8):
+        st, h = as2d_cbuf_create(window)
+        _check(st, "as2d_cbuf_create")
+        self.handle = h
+
+    def publish(self, tokens, request=0, source=0, producer=0, offset=0, time=0.0,
+                confidence=None):
+        rec = as2d_source_record(request, source, producer, offset, time,
+                                 0.0 if confidence is None else confidence,
+                                 0 if confidence is None else 1)
+        _check(as2d_cbuf_publish(self.handle, list(tokens), rec), "as2d_cbuf_publish")
+
+    def candidates(self, b):
+        st, toks = as2d_cbuf_candidates(self.handle, b)
+        _check(st, "as2d_cbuf_candidates")
+        return toks
+
+    def after_call(self, k, n_accepted, correction):
+        _check(as2d_cbuf_after_call(self.handle, k, n_accepted, correction),
+               "as2d_cbuf_after_call")
+
+    def state(self):
+        st, ready, cursor, mode = as2d_cbuf_state(self.handle)
+        _check(st, "as2d_cbuf_state")
+        return ready, cursor, CBUF_MODES[mode]
+
+    def source_of(self, position):
+        st, rec = as2d_cbuf_source_of(self.handle, position)
+        _check(st, "as2d_cbuf_source_of")
+        return {"request": rec.request, "source": rec.source, "producer": rec.producer,
+                "offset": rec.offset, "time": rec.time,
+                "confidence": rec.confidence if rec.has_confidence else None}
+
+    def close(self):
+        if self.handle:
+            as2d_cbuf_free(self.handle)
             self.handle = None
 
     def __del__(self):
@@ -270,6 +395,14 @@ class State:
                               greedy.data_ptr() if greedy is not None else 0,
                               logits.data_ptr() if logits is not None else 0)
         _check(as2d_decode_step(self.handle, out, stream), "as2d_decode_step")
+
+    def verify_from_buffers(self, bufs, b, stream=0):
+        """One verification call with candidates from CandidateBuffer objects
+        (one per request); returns (k_used, committed token lists)."""
+        st, k_used, rows = as2d_verify_from_buffers(
+            self.handle, [x.handle for x in bufs], b, self.batch, stream)
+        _check(st, "as2d_verify_from_buffers")
+        return k_used, rows
 
     def rollback(self, new_len, new_root, stream=0):
         _check(as2d_kv_rollback(self.handle, new_len, new_root, stream), "as2d_kv_rollback")

@@ -9,13 +9,6 @@
 
 using namespace as2d;
 
-struct as2d_model {
-  Model m;
-};
-struct as2d_kv {
-  KvState s;
-};
-
 namespace {
 
 thread_local std::string g_err;
@@ -102,6 +95,9 @@ as2d_status check_config(const as2d_config* c) {
 }
 
 }  // namespace
+
+as2d_status as2d::report_error(as2d_status st, const std::string& msg) { return fail(st, msg); }
+void as2d::clear_error() { g_err.clear(); }
 
 extern "C" const char* as2d_last_error(void) { return g_err.c_str(); }
 
@@ -336,6 +332,8 @@ extern "C" void as2d_kv_free(as2d_kv* kh) {
   for (cudaEvent_t e : kh->s.prof_events) cudaEventDestroy(e);
   cudaFree(kh->s.mk_mem);
   cudaFree(kh->s.work);
+  cudaFree(kh->s.cb_dev);
+  cudaFreeHost(kh->s.cb_host);
   delete kh;
 }
 

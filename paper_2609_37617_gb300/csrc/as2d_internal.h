@@ -182,7 +182,16 @@ struct KvState {
   std::vector<cudaEvent_t> prof_events;  // pairs
   int prof_used = 0;                     // pairs recorded since the last read
   int64_t launches = 0;                  // kernels launched since the last read
+  // staging of as2d_verify_from_buffers (cand_buffer.cu), allocated on first use:
+  // candidates [batch][kMaxK], then n_accepted [batch] and correction [batch]
+  int32_t* cb_dev = nullptr;
+  int32_t* cb_host = nullptr;            // pinned, same layout
 };
+
+// Error reporting shared by the translation units of the C-ABI: records the
+// thread-local message returned by as2d_last_error and passes `st` through.
+as2d_status report_error(as2d_status st, const std::string& msg);
+void clear_error();
 
 // Launchers (k_basic.cu).  All enqueue on `st` and return cudaGetLastError().
 cudaError_t launch_embed(const RowMap& m, const Model& md, KvState& kv,
@@ -224,3 +233,11 @@ cudaError_t launch_f32_from_bf16(float* dst, const void* src, int64_t n,
                                  cudaStream_t st);
 
 }  // namespace as2d
+
+// Handle types of the C-ABI.
+struct as2d_model {
+  as2d::Model m;
+};
+struct as2d_kv {
+  as2d::KvState s;
+};
