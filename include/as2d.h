@@ -231,7 +231,7 @@ void as2d_model_free(as2d_model* model);
 
 /* ---- Candidate buffer, read cursor and alignment -------------------------
    (Section 3.1 "Ordered publication and buffering"; Section 3.2 "Candidate
-   alignment"; App. B.1 "Source records and incremental publication"; App. B.3
+   alignment"; App. C.1 "Source records and incremental publication"; App. C.3
    "Candidate alignment"; Fig. 4.)  Host-side: one buffer per request and
    source.  The producer appends immutable batches of at most
    AS2D_CBUF_BATCH tokens; verification reads a snapshot of what is published
@@ -264,7 +264,7 @@ void as2d_model_free(as2d_model* model);
 #define AS2D_CBUF_REALIGN 1  /* R1/R2: waiting on the token at m          */
 #define AS2D_CBUF_ALONE 2    /* R3: no usable candidates; k = 0           */
 
-/* Source record of one published batch (App. B.1).  confidence is
+/* Source record of one published batch (App. C.1).  confidence is
    meaningful only when has_confidence != 0. */
 typedef struct as2d_source_record {
   int32_t request, source, producer, offset;
@@ -321,6 +321,62 @@ void as2d_cbuf_free(as2d_cbuf* buf);
 as2d_status as2d_verify_from_buffers(as2d_kv* kv, as2d_cbuf* const* bufs, int32_t b,
                                      int32_t* k_used, int32_t* committed,
                                      int32_t* n_committed, void* stream);
+
+/* ---- Producer / verifier sessions and their time accounting --------------
+   (App. D.2 "Overlap, added work, and performance limits": the service
+   intervals, D, V, O, H and the identity T = D + V - O + H;
+   Section 3.1: the producer runs without target feedback and the target
+   never waits for it.) */
+
+/* Service-interval accounting over [0, T].  p: host double [np][2] producer
+   service intervals (start, end); v: host double [nv][2] verifier
+   intervals; each is clipped to [0, T] and merged with the overlapping
+   intervals of its own set.  out: host double [5] receives D = |P|, V = |V|,
+   O = |P n V|, H = |[0, T] \ (P u V)| and T, so that T = D + V - O + H.
+   AS2D_ERR_INVALID_ARG for an interval with end < start, T < 0 or counts
+   < 0. */
+as2d_status as2d_interval_accounting(const double* p, int32_t np, const double* v,
+                                     int32_t nv, double T, double* out);
+
+/* One request decoded to n_commit tokens by a producer publishing into a
+   candidate buffer and a verifier drawing from it. */
+typedef struct as2d_session_spec {
+  as2d_kv* target;        /* batch-1 target state, advanced by the session          */
+  as2d_kv* drafter;       /* batch-1 drafter state, one k = 0 decode step per
+                             produced token on drafter_stream; NULL = no drafter
+                             compute (tokens are published as fast as scripted)  */
+  as2d_cbuf* buf;         /* the request's candidate buffer, written by the session */
+  const int32_t* script;  /* host [n_script]: the token published by producer step i */
+  int32_t n_script;
+  int32_t b;              /* candidates per verification call, 0..AS2D_MAX_K       */
+  int32_t publish_every;  /* producer steps per published batch, 1..AS2D_CBUF_BATCH */
+  int32_t n_commit;       /* stop once at least this many tokens are committed     */
+  int32_t overlapped;     /* 1: the producer runs on its own host thread and stream
+                             alongside the verifier; 0: serial comparator -- the
+                             producer runs (one batch) only while the verifier
+                             waits, whenever fewer than b candidates are ready    */
+  void* target_stream;
+  void* drafter_stream;
+} as2d_session_spec;
+
+typedef struct as2d_session_stats {
+  double T, D, V, O, H;   /* seconds: the accounting above over the session     */
+  int32_t rounds;         /* verification calls (target-only rounds included)   */
+  int32_t alone_rounds;   /* calls with k = 0                                    */
+  int32_t committed;      /* tokens committed (accepted + one per call)          */
+  int32_t accepted;       /* accepted candidates                                 */
+  int32_t producer_steps; /* drafter steps run                                   */
+  int32_t published;      /* tokens published                                    */
+} as2d_session_stats;
+
+/* Run a session.  Producer service intervals are the drafter steps with their
+   publication; verifier intervals are the as2d_verify_from_buffers calls
+   (verification, read-back, alignment).  Blocking; synchronises both
+   streams.  committed: host int32 [n_commit + AS2D_MAX_K + 1] or NULL
+   receives the committed tokens; stats (required) the accounting.  Errors of
+   either side stop the session and are returned. */
+as2d_status as2d_session_run(const as2d_session_spec* spec, int32_t* committed,
+                             as2d_session_stats* stats);
 
 /* Thread-local description of the last error ("" if none). */
 const char* as2d_last_error(void);

@@ -1,7 +1,7 @@
 """Candidate buffer, read cursor and candidate alignment, written from the
 paper (Section 3.1 "Ordered publication and buffering"; Section 3.2
-"Candidate alignment"; App. B.1 "Source records and incremental
-publication"; App. B.3 "Candidate alignment"; Fig. 4).
+"Candidate alignment"; App. C.1 "Source records and incremental
+publication"; App. C.3 "Candidate alignment"; Fig. 4).
 
 TEST INFRASTRUCTURE: plain Python, no shared code with the library's C++
 implementation (csrc/cand_buffer.cu); only tests import it.
@@ -43,7 +43,7 @@ NORMAL, REALIGN, ALONE = "normal", "realign", "alone"
 
 
 class SourceRecord:
-    """App. B.1: request, audio view (source), producer, token offset,
+    """App. C.1: request, audio view (source), producer, token offset,
     publication time, confidence (None when unavailable)."""
 
     def __init__(self, request, source, producer, offset, time, confidence=None):
@@ -81,7 +81,7 @@ class CandidateBuffer:
         return len(self.tokens)
 
     def source_of(self, i):
-        """App. B.1: the source record of the batch that published position i."""
+        """App. C.1: the source record of the batch that published position i."""
         if not 0 <= i < len(self.tokens):
             raise IndexError(i)
         rec = None

@@ -1,7 +1,7 @@
 // cand_buffer.cu -- the candidate buffer, its read cursor and candidate
 // alignment (Section 3.1 "Ordered publication and buffering"; Section 3.2
-// "Candidate alignment"; App. B.1 "Source records and incremental
-// publication"; App. B.3 "Candidate alignment"; Fig. 4), and the verification
+// "Candidate alignment"; App. C.1 "Source records and incremental
+// publication"; App. C.3 "Candidate alignment"; Fig. 4), and the verification
 // call that draws its candidates from such buffers.
 //
 // Host code.  The producer appends immutable batches of at most eight tokens;

@@ -718,13 +718,11 @@ __global__ void __launch_bounds__(128) tc_resid_finish_kernel(const __grid_const
 template <int NB, int EPI>
 cudaError_t tc_gemm_launch(const CUtensorMap& x, const TcParams& p, cudaStream_t st) {
   constexpr uint32_t smem = TcShape<NB>::SMEM;
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(tc_gemm_kernel<NB, EPI>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    attr_set = true;
-  }
+  // set once per instantiation; a function-local static is initialised
+  // exactly once even when several host threads launch at the same time
+  static const cudaError_t attr = cudaFuncSetAttribute(
+      tc_gemm_kernel<NB, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (attr != cudaSuccess) return attr;
   cudaError_t e = launch_pdl(tc_gemm_kernel<NB, EPI>, dim3(p.grid), dim3(192), smem, st, x, p);
   if (e != cudaSuccess || !p.defer || p.grid < 2) return e;
   if (EPI == TC_RESID)

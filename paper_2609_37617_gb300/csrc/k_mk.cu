@@ -500,24 +500,19 @@ __global__ void __launch_bounds__(kMkThreads, 1)
 namespace {
 
 bool mk_enabled() {
-  static int v = -1;
-  if (v < 0) {
+  static const bool v = [] {
     const char* e = getenv("AS2D_PERSISTENT");
-    v = (e && e[0] == '1') ? 1 : 0;
-  }
-  return v == 1;
+    return e && e[0] == '1';
+  }();
+  return v;
 }
 
 template <int NB, int D>
 cudaError_t mk_launch_t(const MkMaps& maps, const MkArgs& a, int grid, cudaStream_t st) {
   constexpr uint32_t smem = MkShape<NB>::SMEM;
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(mk_kernel<NB, D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)smem);
-    if (e != cudaSuccess) return e;
-    attr_set = true;
-  }
+  static const cudaError_t attr_e =
+      cudaFuncSetAttribute(mk_kernel<NB, D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (attr_e != cudaSuccess) return attr_e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
   cfg.blockDim = dim3(kMkThreads);
