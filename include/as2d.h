@@ -315,7 +315,8 @@ void as2d_cbuf_free(as2d_cbuf* buf);
    stream) and reports them to each buffer.  Outputs (host, may be NULL):
    k_used int32 [batch]; committed int32 [batch][b + 1], row r holding the
    request's n_r + 1 committed tokens (accepted candidates, then the
-   correction); n_committed int32 [batch] = n_r + 1.  Device staging memory
+   correction); n_committed int32 [batch] = n_r + 1.  The host's length
+   bounds are tightened with the read-back n_r.  Device staging memory
    is allocated on the first call and kept until as2d_kv_free.  Errors of
    as2d_verify_block are returned as they are, before any buffer changes. */
 as2d_status as2d_verify_from_buffers(as2d_kv* kv, as2d_cbuf* const* bufs, int32_t b,
@@ -372,7 +373,9 @@ typedef struct as2d_session_stats {
 /* Run a session.  Producer service intervals are the drafter steps with their
    publication; verifier intervals are the as2d_verify_from_buffers calls
    (verification, read-back, alignment).  Blocking; synchronises both
-   streams.  committed: host int32 [n_commit + AS2D_MAX_K + 1] or NULL
+   streams, which should be distinct non-default streams for the two sides to
+   overlap on the GPU.  The drafter's capacity must leave room for one
+   position per scripted token.  committed: host int32 [n_commit + AS2D_MAX_K + 1] or NULL
    receives the committed tokens; stats (required) the accounting.  Errors of
    either side stop the session and are returned. */
 as2d_status as2d_session_run(const as2d_session_spec* spec, int32_t* committed,

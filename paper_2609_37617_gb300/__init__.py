@@ -38,7 +38,7 @@ EXPORTED = ("as2d_model_load", "as2d_kv_init_prefilled", "as2d_verify_block",
             "as2d_kv_profile_read", "as2d_decode_step_static", "as2d_cbuf_create",
             "as2d_cbuf_publish", "as2d_cbuf_candidates", "as2d_cbuf_after_call",
             "as2d_cbuf_state", "as2d_cbuf_source_of", "as2d_cbuf_free",
-            "as2d_verify_from_buffers")
+            "as2d_verify_from_buffers", "as2d_interval_accounting", "as2d_session_run")
 KERNEL_CLASSES = {"qkv": 0, "attention": 1, "o": 2, "gate_up": 3, "down": 4,
                   "lm_head": 5, "other": 6, "pass": 7}
 
@@ -67,6 +67,21 @@ class as2d_source_record(ctypes.Structure):
                 ("producer", ctypes.c_int32), ("offset", ctypes.c_int32),
                 ("time", ctypes.c_double), ("confidence", ctypes.c_float),
                 ("has_confidence", ctypes.c_int32)]
+
+
+class as2d_session_spec(ctypes.Structure):
+    _fields_ = [("target", ctypes.c_void_p), ("drafter", ctypes.c_void_p),
+                ("buf", ctypes.c_void_p), ("script", ctypes.c_void_p),
+                ("n_script", ctypes.c_int32), ("b", ctypes.c_int32),
+                ("publish_every", ctypes.c_int32), ("n_commit", ctypes.c_int32),
+                ("overlapped", ctypes.c_int32), ("target_stream", ctypes.c_void_p),
+                ("drafter_stream", ctypes.c_void_p)]
+
+
+class as2d_session_stats(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_double) for n in ("T", "D", "V", "O", "H")] + \
+               [(n, ctypes.c_int32) for n in ("rounds", "alone_rounds", "committed", "accepted",
+                                              "producer_steps", "published")]
 
 
 _P = ctypes.c_void_p
@@ -115,6 +130,11 @@ for _n in ("as2d_cbuf_create", "as2d_cbuf_publish", "as2d_cbuf_candidates",
            "as2d_cbuf_after_call", "as2d_cbuf_state", "as2d_cbuf_source_of",
            "as2d_verify_from_buffers"):
     getattr(_lib, _n).restype = _S
+_lib.as2d_interval_accounting.argtypes = [_P, _S, _P, _S, ctypes.c_double, _P]
+_lib.as2d_interval_accounting.restype = _S
+_lib.as2d_session_run.argtypes = [ctypes.POINTER(as2d_session_spec), _P,
+                                  ctypes.POINTER(as2d_session_stats)]
+_lib.as2d_session_run.restype = _S
 _lib.as2d_last_error.argtypes = []
 _lib.as2d_last_error.restype = ctypes.c_char_p
 
@@ -286,6 +306,38 @@ def as2d_verify_from_buffers(kv, bufs, b, batch, stream=0):
     st = _lib.as2d_verify_from_buffers(kv, hb, b, k_used, comm, ncomm, stream)
     rows = [list(comm[r * (b + 1): r * (b + 1) + ncomm[r]]) for r in range(batch)]
     return st, list(k_used), rows
+
+
+def as2d_interval_accounting(p, v, T):
+    """p, v: lists of (start, end).  Returns (status, [D, V, O, H, T])."""
+    pa = (ctypes.c_double * max(2 * len(p), 1))(*[x for iv in p for x in iv])
+    va = (ctypes.c_double * max(2 * len(v), 1))(*[x for iv in v for x in iv])
+    out = (ctypes.c_double * 5)()
+    st = _lib.as2d_interval_accounting(pa, len(p), va, len(v), T, out)
+    return st, list(out)
+
+
+def as2d_session_run(spec, n_commit, b):
+    """Returns (status, committed list, stats dict)."""
+    comm = (ctypes.c_int32 * (n_commit + AS2D_MAX_K + 1))()
+    stats = as2d_session_stats()
+    st = _lib.as2d_session_run(ctypes.byref(spec), comm, ctypes.byref(stats))
+    d = {n: getattr(stats, n) for n, _ in as2d_session_stats._fields_}
+    return st, list(comm[:max(stats.committed, 0)]), d
+
+
+def session_run(target, drafter, buf, script, b, n_commit, overlapped, publish_every=8,
+                target_stream=0, drafter_stream=0):
+    """Run a producer/verifier session (as2d_session_run) on State objects and
+    a CandidateBuffer; returns (committed tokens, stats dict)."""
+    arr = _i32_array(script) if len(script) else None
+    spec = as2d_session_spec(target.handle, drafter.handle if drafter is not None else None,
+                             buf.handle, ctypes.cast(arr, ctypes.c_void_p) if arr else None,
+                             len(script), b, publish_every, n_commit, int(bool(overlapped)),
+                             target_stream, drafter_stream)
+    st, comm, stats = as2d_session_run(spec, n_commit, b)
+    _check(st, "as2d_session_run")
+    return comm, stats
 
 
 def exported_symbols():

@@ -283,6 +283,7 @@ extern "C" as2d_status as2d_verify_from_buffers(as2d_kv* kh, as2d_cbuf* const* b
     if (n_committed) n_committed[r] = n + 1;
     if (k_used) k_used[r] = k[r];
     bufs[r]->b.after_call(k[r], n, h_corr[r]);
+    s.len_upper[r] -= k[r] - n;  // the call grew the length by n + 1, not k + 1
     off += k[r];
   }
   return AS2D_OK;

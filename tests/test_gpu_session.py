@@ -143,3 +143,49 @@ def test_empty_buffer_is_plain_decoding(pair):
         assert k_used == [0] and len(rows[0]) == 1
     assert buf.state()[2] in ("realign", "alone")
     st.close()
+
+
+def _run_session(lib, pair, drafter, root, script, overlapped, n_commit):
+    import torch
+    st = pair.state([L0], CAP, [root])
+    dst = drafter.state([L0], CAP, [int(W.root_tokens(drafter.cfg, 1, 1)[0])])
+    s_t, s_d = torch.cuda.Stream(), torch.cuda.Stream()
+    buf = lib.CandidateBuffer(8)
+    comm, stats = lib.session_run(st, dst, buf, script, 8, n_commit, overlapped,
+                                  target_stream=s_t.cuda_stream, drafter_stream=s_d.cuda_stream)
+    ln, rt = st.read_state()
+    assert ln == [L0 + len(comm)] and rt == [comm[-1]]
+    st.check()
+    dst.check()
+    st.close()
+    dst.close()
+    return comm, stats
+
+
+def test_session_runner_serial_and_overlapped(pair):
+    """as2d_session_run with a drafter decoding on its own stream: both
+    schedules commit the target's greedy text, and the accounting satisfies
+    T = D + V - O + H with no overlap in the serial comparator."""
+    import paper_2609_37617_gb300 as lib
+    cfg = pair.cfg
+    drafter = Pair(W.TINY, seed=1)
+    root = int(W.root_tokens(cfg, 1, 0)[0])
+    oc = pair.oracle_cache(L0, CAP)
+    cont, margins = oracle.greedy_continuation(pair.oracle, oc, L0, root, N_TOK + 24)
+    script = _producer(cont, 9, cfg.vocab)[:N_TOK + 16]
+    sure = _sure_prefix(margins)
+    runs = {}
+    for overlapped in (False, True):
+        comm, stats = _run_session(lib, pair, drafter, root, script, overlapped, N_TOK)
+        assert len(comm) >= N_TOK and len(comm) == stats["committed"]
+        m = min(sure, len(comm))
+        assert comm[:m] == [int(t) for t in cont[:m]]
+        T, D, V, O, H = (stats[x] for x in "TDVOH")
+        assert abs(D + V - O + H - T) < 1e-9 * max(T, 1.0)
+        assert 0 <= O <= min(D, V) + 1e-12 and T >= max(D, V) + H - 1e-9
+        assert stats["accepted"] == stats["committed"] - stats["rounds"]
+        assert stats["producer_steps"] == stats["published"] <= len(script)
+        runs[overlapped] = (comm, stats)
+    assert runs[False][1]["O"] == 0.0
+    n = min(len(runs[False][0]), len(runs[True][0]))
+    assert runs[False][0][:n] == runs[True][0][:n]
