@@ -60,9 +60,10 @@ def parse():
                          "k + 1 <= 32 rows), else gate_up")
     ap.add_argument("--model", default="7b", help="model shape (7b; smaller ones for quick checks)")
     ap.add_argument("--kv-len", type=int, default=1564)
-    ap.add_argument("--sweep", default="0,1,2,4,8,16",
-                    help="block sizes k for the verify-time sweep ('' to skip)")
-    ap.add_argument("--sweep-blocks", type=int, default=32)
+    ap.add_argument("--sweep", default=",".join(str(i) for i in range(17)),
+                    help="block sizes k for the verify-time sweep ('' to skip); the budget "
+                         "selection needs all of 0..16")
+    ap.add_argument("--sweep-blocks", type=int, default=24)
     ap.add_argument("--session", action="store_true",
                     help="producer/verifier session line instead of the verify-step line")
     ap.add_argument("--drafter", default="1.5b", help="drafter model shape for --session")
@@ -345,6 +346,10 @@ def run_ours(args, ws, rank, local):
                 for e in sweep:
                     e["R_pct"] = round(100.0 * (1.0 - e["verify_us_mean"] / (e["K"] * v1)), 1)
 
+        budget = None
+        if len(sweep) == 17 and [e["k"] for e in sweep] == list(range(17)):
+            budget = select_budget(args, lib, state, traj, sweep, cfg, L0, root0, sh)
+
         e2e = None
         if not args.no_e2e:
             e2e = run_e2e(args, lib, W, state, traj, plans, cfg, L0, root0, sh, stream)
@@ -409,6 +414,7 @@ def run_ours(args, ws, rank, local):
                                "builder kernels (test input) in the timed pass",
         "class_us_per_block": breakdown,
         "k_sweep": sweep,
+        "budget": budget,
         "clocks": clk,
         "e2e": e2e,
     }
@@ -420,6 +426,50 @@ def run_ours(args, ws, rank, local):
     model.close()
     if ws > 1:
         dist.destroy_process_group()
+
+
+def select_budget(args, lib, state, traj, sweep, cfg, L0, root0, sh):
+    """Offline budget choice (Section 3.3; App. D.2): the measured mean call
+    time of every k and development traces -- windows of the target's greedy
+    text, the producer's copy with each token substituted w.p. 0.25 (the
+    acceptance of this workload) -- rank b = 0..16 by estimated committed
+    tok/s (as2d_budget_select).  The chosen b and b = 8 are then run as real
+    sessions through the candidate buffer (producer text published ahead, no
+    drafter cost) and measured."""
+    rng = np.random.default_rng(args.seed + 4242)
+    traj_h = [int(x) for x in traj.cpu().numpy()[1:]]
+    win, n_commit = 220, 180
+    traces = []
+    for w in range(min(4, len(traj_h) // win)):
+        ref = traj_h[w * win:(w + 1) * win]
+        prod = [int(rng.integers(cfg.vocab)) if rng.random() < 0.25 else t for t in ref]
+        traces.append((ref, prod))
+    if not traces:
+        return None
+    cost = [e["verify_us_mean"] for e in sweep]
+    st, best, tok_s, calls = lib.as2d_budget_select(cost, traces, n_commit, 8, 16)
+    lib._check(st, "as2d_budget_select")
+    measured = {}
+    ref, prod = traces[0]
+    for b in sorted({best, 8}):
+        state.rollback([L0], [root0], sh)
+        state.read_state(sh)
+        buf = lib.CandidateBuffer(8)
+        comm, stats = lib.session_run(state, None, buf, prod, b, n_commit, False,
+                                      target_stream=sh)
+        assert comm[:len(ref)] == ref[:len(comm)], "session text differs from greedy decoding"
+        measured[str(b)] = {"tok_s": round(stats["committed"] / stats["V"], 1),
+                            "calls": stats["rounds"], "committed": stats["committed"]}
+    state.check(sh)
+    v1 = cost[0]
+    return {"selected_b": best,
+            "est_tok_s": [round(x, 1) for x in tok_s],
+            "est_calls": calls,
+            "R_pct": [round(100.0 * (1.0 - c / ((k + 1) * v1)), 1) for k, c in enumerate(cost)],
+            "measured_first_trace": measured,
+            "dev": f"{len(traces)} windows of {win} greedy tokens, producer substitution "
+                   f"p=0.25, {n_commit} committed per window, window W=8",
+            "measured_note": "verifier service time only (producer text published ahead)"}
 
 
 def run_e2e(args, lib, W, state, traj, plans, cfg, L0, root0, sh, stream):

@@ -381,6 +381,33 @@ typedef struct as2d_session_stats {
 as2d_status as2d_session_run(const as2d_session_spec* spec, int32_t* committed,
                              as2d_session_stats* stats);
 
+/* ---- Offline budget selection -----------------------------------------------
+   (Section 3.3 "Device-profiled configuration": device cost profiles and
+   development traces choose one fixed proposal budget b; App. B, Eq. for
+   R(K), the per-position cost reduction of width K; App. D.2 "Fixed
+   configurations and development splits": budgets ranked by pooled
+   throughput.) */
+
+/* Estimate the pooled committed tokens per second of every budget b in
+   0..b_max on development traces.  Each trace is replayed with the alignment
+   rules above: the producer's whole text is published before the first call
+   (in AS2D_CBUF_BATCH-token batches), each call takes up to b candidates,
+   the target commits the trace's reference text (accepting the longest
+   matching prefix, then one token) until n_commit tokens are committed, and
+   each call of k candidates is charged cost_us[k].
+   cost_us: host double [AS2D_MAX_K + 1], mean call time by k (> 0).
+   refs, prods: host int32, the traces' reference and producer texts
+   concatenated, with lengths ref_len, prod_len host int32 [n_traces];
+   ref_len[t] >= n_commit + b_max + 1.  window: the alignment search bound.
+   Outputs (host): tok_s double [b_max + 1]; calls int32 [b_max + 1] (may be
+   NULL), the pooled call counts; *best_b, the budget with the highest
+   estimate (the smallest such b on ties). */
+as2d_status as2d_budget_select(const double* cost_us, const int32_t* refs,
+                               const int32_t* ref_len, const int32_t* prods,
+                               const int32_t* prod_len, int32_t n_traces,
+                               int32_t n_commit, int32_t window, int32_t b_max,
+                               double* tok_s, int32_t* calls, int32_t* best_b);
+
 /* Thread-local description of the last error ("" if none). */
 const char* as2d_last_error(void);
 

@@ -38,7 +38,8 @@ EXPORTED = ("as2d_model_load", "as2d_kv_init_prefilled", "as2d_verify_block",
             "as2d_kv_profile_read", "as2d_decode_step_static", "as2d_cbuf_create",
             "as2d_cbuf_publish", "as2d_cbuf_candidates", "as2d_cbuf_after_call",
             "as2d_cbuf_state", "as2d_cbuf_source_of", "as2d_cbuf_free",
-            "as2d_verify_from_buffers", "as2d_interval_accounting", "as2d_session_run")
+            "as2d_verify_from_buffers", "as2d_interval_accounting", "as2d_session_run",
+            "as2d_budget_select")
 KERNEL_CLASSES = {"qkv": 0, "attention": 1, "o": 2, "gate_up": 3, "down": 4,
                   "lm_head": 5, "other": 6, "pass": 7}
 
@@ -135,6 +136,8 @@ _lib.as2d_interval_accounting.restype = _S
 _lib.as2d_session_run.argtypes = [ctypes.POINTER(as2d_session_spec), _P,
                                   ctypes.POINTER(as2d_session_stats)]
 _lib.as2d_session_run.restype = _S
+_lib.as2d_budget_select.argtypes = [_P, _P, _P, _P, _P, _S, _S, _S, _S, _P, _P, _P]
+_lib.as2d_budget_select.restype = _S
 _lib.as2d_last_error.argtypes = []
 _lib.as2d_last_error.restype = ctypes.c_char_p
 
@@ -338,6 +341,25 @@ def session_run(target, drafter, buf, script, b, n_commit, overlapped, publish_e
     st, comm, stats = as2d_session_run(spec, n_commit, b)
     _check(st, "as2d_session_run")
     return comm, stats
+
+
+def as2d_budget_select(cost_us, traces, n_commit, window, b_max):
+    """cost_us: AS2D_MAX_K + 1 mean call times by k; traces: list of
+    (reference text, producer text).  Returns (status, best b, tok/s per b,
+    calls per b)."""
+    cost = (ctypes.c_double * (AS2D_MAX_K + 1))(*[float(c) for c in cost_us])
+    refs = [int(t) for r, _ in traces for t in r]
+    prods = [int(t) for _, p in traces for t in p]
+    ra = _i32_array(refs or [0])
+    pa = _i32_array(prods or [0])
+    rl = _i32_array([len(r) for r, _ in traces] or [0])
+    pl = _i32_array([len(p) for _, p in traces] or [0])
+    tok_s = (ctypes.c_double * (max(b_max, 0) + 1))()
+    calls = (ctypes.c_int32 * (max(b_max, 0) + 1))()
+    best = ctypes.c_int32(-1)
+    st = _lib.as2d_budget_select(cost, ra, rl, pa, pl, len(traces), n_commit, window, b_max,
+                                 tok_s, calls, ctypes.byref(best))
+    return st, best.value, list(tok_s), list(calls)
 
 
 def exported_symbols():
