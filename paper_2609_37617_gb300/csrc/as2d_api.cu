@@ -315,10 +315,15 @@ extern "C" as2d_status as2d_kv_init_prefilled(as2d_model* mh, int32_t batch,
     return fail(AS2D_ERR_CUDA, std::string("preparing the persistent pass: ") + cudaGetErrorString(e));
   }
   e = cudaMemset(s.work, 0, bytes);
+  if (e == cudaSuccess)
+    e = cudaMalloc(&s.rope_full, (size_t)capacity * (m.cfg.head_dim / 2) * sizeof(float2));
+  if (e == cudaSuccess) e = launch_rope_table(m, s, 0);
   if (e == cudaSuccess) e = cudaMemcpy(s.d_len, kv_len, batch * 4, cudaMemcpyHostToDevice);
   if (e == cudaSuccess) e = cudaMemcpy(s.d_root, root_tokens, batch * 4, cudaMemcpyHostToDevice);
   if (e == cudaSuccess) e = cudaDeviceSynchronize();
   if (e != cudaSuccess) {
+    cudaFree(s.rope_full);
+    cudaFree(s.mk_mem);
     cudaFree(s.work);
     delete kh;
     return fail(AS2D_ERR_CUDA, std::string("initialising the state: ") + cudaGetErrorString(e));
@@ -332,6 +337,7 @@ extern "C" void as2d_kv_free(as2d_kv* kh) {
   for (cudaEvent_t e : kh->s.prof_events) cudaEventDestroy(e);
   cudaFree(kh->s.mk_mem);
   cudaFree(kh->s.work);
+  cudaFree(kh->s.rope_full);
   cudaFree(kh->s.cb_dev);
   cudaFreeHost(kh->s.cb_host);
   delete kh;
@@ -400,8 +406,8 @@ cudaError_t tc_project(int epi, const Model& m, KvState& s, const RowMap& rm, co
   //   at least as many tiles as SMs (gate/up): whole tiles per CTA, as
   //     evenly as they go, each finished by its own CTA;
   //   otherwise stream-K over one CTA per SM; residual projections leave
-  //     their split tiles to tc_reduce_kernel, the LM head finishes them in
-  //     the GEMM (last CTA of a tile).
+  //     their split tiles to tc_resid_finish_kernel, the LM head finishes
+  //     them in the GEMM (last CTA of a tile).
   p.grid = (int)(p.units < m.sm_count ? p.units : m.sm_count);
   p.split = 0;
   p.defer = epi == TC_RESID ? 1 : 0;

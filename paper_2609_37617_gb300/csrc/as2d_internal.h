@@ -156,6 +156,7 @@ struct KvState {
   bf16* u = nullptr;         // [2 rows][F] SwiGLU output
   unsigned long long* best = nullptr;  // [rows] packed (logit, index) maxima
   float2* rope = nullptr;    // [rows][d/2] (cos, sin) at each row's position
+  float2* rope_full = nullptr;  // [capacity][d/2] (cos, sin) of every position (own allocation)
   int rows_alloc = 0;        // activation rows allocated (>= every NB used)
   int nb_max = 16;
   float* ws = nullptr;       // [sm_count][2][nb_max][128] partial GEMM tiles
@@ -201,6 +202,8 @@ cudaError_t launch_accept(const RowMap& m, const Model& md, KvState& kv,
                           cudaStream_t st);
 cudaError_t launch_rollback(KvState& kv, const int32_t* new_len,
                             const int32_t* new_root, cudaStream_t st);
+// Fills kv.rope_full for positions [0, capacity).
+cudaError_t launch_rope_table(const Model& md, KvState& kv, cudaStream_t st);
 // Load-time weight re-layout (k_pack.cu).
 size_t packed_elems(int n_rows, int K);
 cudaError_t pack_weights(bf16* dst, int n_rows, int K, const void* const* segs,

@@ -15,7 +15,7 @@
 // Pass 1 (attn_part_kernel): one CTA per (64-key partition, kv head, request).
 // Keys and values are staged in shared memory -- those already in the cache
 // before the kernel waits for pass 0, the block's own after; each warp takes
-// 16 query rows;
+// 16 query rows at a time (4 to 8 warps, by the largest request);
 // S = Q K^T and O = P V run on the tensor cores (mma.sync m16n8k16, bf16 in,
 // fp32 accumulate), with Q and P each split into bf16 hi + lo parts (two MMAs)
 // so that only the bf16 cache itself limits precision; the softmax runs in
@@ -120,15 +120,31 @@ cudaError_t launch_attention_split(const RowMap& m, const Model& md, KvState& kv
   a.qkv_split = kv.qkv_split;
   a.qkv_ld = kv.rows_alloc;
   const dim3 gf(m.rows, c.n_q_heads + 2 * c.n_kv_heads);
+  // Eight warps stage a partition fastest; when there are more items than
+  // SMs, one warp per 16 query rows of the largest request (at least four,
+  // for the staging copies) lets two CTAs share an SM, so long prefixes need
+  // half the waves.  Which warp takes a row tile does not change its
+  // arithmetic.
+  int warps = 8;
+  if ((long long)parts * c.n_kv_heads * kv.batch > md.sm_count) {
+    int qn_max = 0;
+    for (int b = 0; b < kv.batch; ++b) {
+      const int qn = (m.start[b + 1] - m.start[b]) * (c.n_q_heads / c.n_kv_heads);
+      qn_max = qn > qn_max ? qn : qn_max;
+    }
+    warps = (qn_max + 15) / 16;
+    warps = warps < 4 ? 4 : (warps > 8 ? 8 : warps);
+  }
+  const dim3 tpart(32 * warps);
   cudaError_t e;
   kv.launches += 3;
   if (c.head_dim == 128) {
     e = launch_pdl(qkv_finish_kernel<128>, gf, dim3(64), 0, st, a);
-    if (e == cudaSuccess) e = launch_pdl(attn_part_kernel<128>, g1, dim3(256), 0, st, a);
+    if (e == cudaSuccess) e = launch_pdl(attn_part_kernel<128>, g1, tpart, 0, st, a);
     if (e == cudaSuccess) e = launch_pdl(attn_merge_kernel<128>, g2, dim3(128), 0, st, a);
   } else {
     e = launch_pdl(qkv_finish_kernel<64>, gf, dim3(32), 0, st, a);
-    if (e == cudaSuccess) e = launch_pdl(attn_part_kernel<64>, g1, dim3(256), 0, st, a);
+    if (e == cudaSuccess) e = launch_pdl(attn_part_kernel<64>, g1, tpart, 0, st, a);
     if (e == cudaSuccess) e = launch_pdl(attn_merge_kernel<64>, g2, dim3(64), 0, st, a);
   }
   return e;

@@ -16,13 +16,29 @@ namespace {
 
 // ---- embedding gather --------------------------------------------------------
 
-// Also writes the row's rotary table: (cos, sin) of pos * theta^(-2e/d) for
-// e < d/2, angles and trigonometry in double, rounded once to float.
+// (cos, sin) of pos * theta^(-2e/d), e < d/2: angle and trigonometry in
+// double, rounded once to float.
+__device__ __forceinline__ float2 rope_angle(int pos, int e, int d, double theta) {
+  const double ang = (double)pos * pow(theta, -2.0 * (double)e / (double)d);
+  double sn, cs;
+  sincos(ang, &sn, &cs);
+  return make_float2((float)cs, (float)sn);
+}
+
+// The rotary table of every position of a state, built once at set-up.
+__global__ void rope_table_kernel(float2* __restrict__ out, int d, double theta) {
+  const int pos = blockIdx.x, e = threadIdx.x;
+  out[(size_t)pos * (d / 2) + e] = rope_angle(pos, e, d, theta);
+}
+
+// Also writes the row's rotary table -- gathered from the state's table of
+// every position when there is one (rope_full), else computed.
 __global__ void __launch_bounds__(128) embed_kernel(
     RowMap m, const int32_t* __restrict__ cand, const int32_t* __restrict__ root,
     const bf16* __restrict__ E, int H, int V, float* __restrict__ h, int32_t* err, int32_t* bad,
-    const int32_t* __restrict__ len, float2* __restrict__ rope, int d, double theta,
-    const float* __restrict__ g0, bf16* __restrict__ xn, float* __restrict__ ss, int ss_ld) {
+    const int32_t* __restrict__ len, float2* __restrict__ rope, const float2* __restrict__ rope_full,
+    int d, double theta, const float* __restrict__ g0, bf16* __restrict__ xn,
+    float* __restrict__ ss, int ss_ld) {
   ptx::griddep_wait();
   ptx::griddep_launch_dependents();
   __shared__ float part[4];
@@ -30,11 +46,9 @@ __global__ void __launch_bounds__(128) embed_kernel(
   const int b = row_request(m, r);
   const int i = r - m.start[b];
   if ((int)threadIdx.x < d / 2) {
-    const int e = threadIdx.x;
-    const double ang = (double)(len[b] + i) * pow(theta, -2.0 * (double)e / (double)d);
-    double sn, cs;
-    sincos(ang, &sn, &cs);
-    rope[(size_t)r * (d / 2) + e] = make_float2((float)cs, (float)sn);
+    const int e = threadIdx.x, pos = len[b] + i;
+    rope[(size_t)r * (d / 2) + e] =
+        rope_full ? rope_full[(size_t)pos * (d / 2) + e] : rope_angle(pos, e, d, theta);
   }
   int tok = (i == 0) ? root[b] : cand[m.start[b] - b + i - 1];
   if (tok < 0 || tok >= V) {
@@ -93,8 +107,14 @@ cudaError_t launch_embed(const RowMap& m, const Model& md, KvState& kv,
   return launch_pdl(embed_kernel, dim3(m.rows), dim3(128), 0, st, m, cand,
                     (const int32_t*)kv.d_root, (const bf16*)md.embed, md.cfg.hidden,
                     md.cfg.vocab, kv.h, kv.d_err, kv.d_err + 1, (const int32_t*)kv.d_len,
-                    kv.rope, md.cfg.head_dim, (double)md.cfg.rope_theta, md.attn_norm[0], kv.xn,
-                    kv.ss, kv.rows_alloc);
+                    kv.rope, (const float2*)kv.rope_full, md.cfg.head_dim,
+                    (double)md.cfg.rope_theta, md.attn_norm[0], kv.xn, kv.ss, kv.rows_alloc);
+}
+
+cudaError_t launch_rope_table(const Model& md, KvState& kv, cudaStream_t st) {
+  rope_table_kernel<<<kv.capacity, md.cfg.head_dim / 2, 0, st>>>(
+      kv.rope_full, md.cfg.head_dim, (double)md.cfg.rope_theta);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_accept(const RowMap& m, const Model& md, KvState& kv,
