@@ -353,10 +353,12 @@ __device__ __forceinline__ void tc_reduce_tile(const TcParams& p, float* sC, flo
           const int cp = c_first + part0 + pp;
           // slot 1 holds a CTA's last segment when it began in an earlier tile
           const int sl = (cp == c_first && (int)(tc_start(cp, p) / p.kb) != tile) ? 1 : 0;
-          const float* src = p.ws + ((size_t)(cp * 2 + sl) * 128 + nl) * NB + ch * CH;
+          const float* src = p.ws + ((size_t)(cp * 2 + sl) * NB + ch * CH) * 128 + nl;
 #pragma unroll
           for (int q = 0; q < 4; ++q)
-            if (4 * q < live) v[pp][q] = __ldcg(reinterpret_cast<const float4*>(src) + q);
+            if (4 * q < live)
+              v[pp][q] = make_float4(__ldcg(src + (4 * q) * 128), __ldcg(src + (4 * q + 1) * 128),
+                                     __ldcg(src + (4 * q + 2) * 128), __ldcg(src + (4 * q + 3) * 128));
         }
       }
       if (part0 == 0) {
@@ -600,16 +602,14 @@ __global__ void __launch_bounds__(192, 1)
         if (lane == 0) ptx::mbar_arrive(&acc_empty[buf]);
       } else {
         const int slot = (tile == first_tile) ? 0 : 1;
-        // partial tile, laid out [n][NB]: a thread's token rows are contiguous
-        float* wsp = p.ws + ((size_t)(c * 2 + slot) * 128 + nl) * NB;
+        // partial tile, laid out [NB][128]: a warp's stores of one token row
+        // are 32 consecutive floats, and so are the finishing loads
+        float* wsp = p.ws + (size_t)(c * 2 + slot) * NB * 128 + nl;
         for (int ch = 0; ch < nchunks; ++ch) {
           uint32_t v[16];
           tc_load_acc<NB>(tbase, ch, v);
 #pragma unroll
-          for (int q = 0; q < 4; ++q)
-            *reinterpret_cast<float4*>(wsp + ch * CH + 4 * q) =
-                make_float4(__uint_as_float(v[4 * q]), __uint_as_float(v[4 * q + 1]),
-                            __uint_as_float(v[4 * q + 2]), __uint_as_float(v[4 * q + 3]));
+          for (int j = 0; j < 16; ++j) wsp[(size_t)(ch * CH + j) * 128] = __uint_as_float(v[j]);
         }
         ptx::tc_fence_before();
         __syncwarp();
@@ -694,7 +694,7 @@ __global__ void __launch_bounds__(128) tc_resid_finish_kernel(const __grid_const
       if (part0 + pp < nparts) {
         const int cp = c_first + part0 + pp;
         const int sl = (cp == c_first && (int)(tc_start(cp, p) / p.kb) != tile) ? 1 : 0;
-        v[pp] = __ldcg(p.ws + ((size_t)(cp * 2 + sl) * 128 + n) * NB + m);
+        v[pp] = __ldcg(p.ws + ((size_t)(cp * 2 + sl) * NB + m) * 128 + n);
       }
     }
 #pragma unroll

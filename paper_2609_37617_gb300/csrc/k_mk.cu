@@ -430,15 +430,12 @@ __global__ void __launch_bounds__(kMkThreads, 1)
             if (lane == 0) ptx::mbar_arrive(&acc_empty[buf]);
           } else {
             const int slot = (tile == first_tile) ? 0 : 1;
-            float* wsp = p.ws + ((size_t)(c * 2 + slot) * 128 + nl) * NB;
+            float* wsp = p.ws + (size_t)(c * 2 + slot) * NB * 128 + nl;  // [NB][128]
             for (int ch = 0; ch < nchunks; ++ch) {
               uint32_t v[16];
               tc_load_acc<NB>(tbase, ch, v);
 #pragma unroll
-              for (int q = 0; q < 4; ++q)
-                *reinterpret_cast<float4*>(wsp + ch * CH + 4 * q) =
-                    make_float4(__uint_as_float(v[4 * q]), __uint_as_float(v[4 * q + 1]),
-                                __uint_as_float(v[4 * q + 2]), __uint_as_float(v[4 * q + 3]));
+              for (int j = 0; j < 16; ++j) wsp[(size_t)(ch * CH + j) * 128] = __uint_as_float(v[j]);
             }
             ptx::tc_fence_before();
             __syncwarp();
