@@ -41,7 +41,7 @@ WORKLOAD = "7b"
 # of the kernel as it stands (profiles/); None once the kernel has changed.
 # dram bytes per launch from an ncu capture of the current kernel; None when
 # the kernel changed after the capture
-TRAFFIC = {"gate_up": 275081216}  # 271,881,472 read + 3,199,744 written
+TRAFFIC = {"gate_up": 275262720}  # 271,890,688 read + 3,372,032 written
 
 
 def parse():
@@ -417,7 +417,8 @@ def run_ours(args, ws, rank, local):
         "config": {"workload": f"{args.model} verify, k={k}, L0={L0}, {steps} consecutive blocks, "
                                "geometric acceptance (mean 3, capped at k)",
                    "k": k, "kv_len": L0, "blocks": steps, "batch": 1,
-                   "l2": "inputs larger than L2 (14.1 GB of weights streamed per step)",
+                   "l2": f"inputs larger than L2 ({cfg.weight_bytes() / 1e9:.2f} GB of weights "
+                         "streamed per step)",
                    "parallelism": f"replicas x{ws}" if ws > 1 else "single GPU"},
         "verify_us": {"median": round(med_us, 1), "p10": round(float(np.percentile(per_block_us, 10)), 1),
                       "p90": round(float(np.percentile(per_block_us, 90)), 1)},
