@@ -365,6 +365,7 @@ def run_ours(args, ws, rank, local):
         e2e = None
         if not args.no_e2e:
             e2e = run_e2e(args, lib, W, state, traj, plans, cfg, L0, root0, sh, stream)
+        prefill = measure_prefill(args, lib, W, state, cfg, L0, root0, sh, stream)
 
     if ws > 1:
         elapsed_ms, committed_all = reduce_ranks(elapsed_ms, committed, "cuda")
@@ -432,6 +433,7 @@ def run_ours(args, ws, rank, local):
         "class_us_per_block": breakdown,
         "k_sweep": sweep,
         "budget": budget,
+        "prefill": prefill,
         "clocks": clk,
         "e2e": e2e,
     }
@@ -443,6 +445,34 @@ def run_ours(args, ws, rank, local):
     model.close()
     if ws > 1:
         dist.destroy_process_group()
+
+
+def measure_prefill(args, lib, W, state, cfg, L0, root0, sh, stream, n_instr=64, reps=5):
+    """Instruction-suffix prefill (App. A.1): the last n_instr positions of the
+    workload's prefix forwarded by as2d_prefill over the retained audio
+    positions before them (CUDA events on the launching stream; after every
+    other measurement, since it rewrites those cache entries)."""
+    import torch
+    audio = L0 - n_instr
+    tok = torch.from_numpy(W.instruction_tokens(cfg, n_instr, args.seed)).cuda()
+    first = torch.zeros(1, dtype=torch.int32, device="cuda")
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    times = []
+    for r in range(reps + 1):
+        state.rollback([audio], [root0], sh)
+        state.read_state(sh)
+        t0.record(stream)
+        state.prefill(tok, first, sh)
+        t1.record(stream)
+        torch.cuda.synchronize()
+        if r > 0:
+            times.append(t0.elapsed_time(t1))
+    state.check(sh)
+    ms = float(np.mean(times))
+    return {"tokens": n_instr, "audio_positions": audio, "ms": round(ms, 3),
+            "tok_s": round(n_instr / (ms / 1e3), 1),
+            "calls": -(-n_instr // 17), "reps": reps}
 
 
 def select_budget(args, lib, state, traj, sweep, cfg, L0, root0, sh):

@@ -140,6 +140,20 @@ as2d_status as2d_verify_block(as2d_kv* kv, const int32_t* candidates,
                               const int32_t* k, const as2d_verify_out* out,
                               void* stream);
 
+/* Instruction-suffix prefill (App. A.1: processing the instruction with the
+   retained, compatible audio KV gives the initial decoding state): forwards
+   tokens[0..n) (device int32 [n], ids in [0, vocab)) at positions
+   L .. L + n - 1 of a batch-1 state and keeps every entry, in chunks of at
+   most AS2D_MAX_K + 1 rows through the verification pass.  The pending root
+   before the call is discarded; afterwards L' = L + n and the root is the
+   greedy token after tokens[n - 1] -- the first token of the response --
+   also written to first_token (device int32 [1]) unless it is NULL.
+   AS2D_ERR_UNSUPPORTED for batch > 1, AS2D_ERR_CAPACITY when the length
+   bound plus n exceeds the capacity; bad token ids are device errors
+   (as2d_kv_check).  Asynchronous on `stream`. */
+as2d_status as2d_prefill(as2d_kv* kv, const int32_t* tokens, int32_t n,
+                         int32_t* first_token, void* stream);
+
 /* One greedy decode step for every request: as2d_verify_block with all
    k_b = 0 (App. C.2: with no ready candidate the target advances alone by one
    token). */

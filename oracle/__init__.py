@@ -228,3 +228,17 @@ def greedy_continuation(model, cache, length, root, n):
         margins.append(m)
         toks.append(tok)
     return np.array(toks[:n], dtype=np.int32), np.array(margins)
+
+
+def prefill(model, cache, length, tokens):
+    """Instruction-suffix prefill (App. A.1): the tokens forwarded one greedy
+    decode step at a time after the `length` retained positions (Eq. 3), their
+    keys and values appended to `cache` in place.  Returns (the first token of
+    the response -- the greedy token after the last one --, its margin, the
+    last row's logits)."""
+    logits = None
+    for i, t in enumerate(tokens):
+        logits = model.decode_step(cache, length + i, int(t))
+    tok, m = argmax(logits)
+    return tok, m, logits
+

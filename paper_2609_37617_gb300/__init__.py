@@ -39,7 +39,7 @@ EXPORTED = ("as2d_model_load", "as2d_kv_init_prefilled", "as2d_verify_block",
             "as2d_cbuf_publish", "as2d_cbuf_candidates", "as2d_cbuf_after_call",
             "as2d_cbuf_state", "as2d_cbuf_source_of", "as2d_cbuf_free",
             "as2d_verify_from_buffers", "as2d_interval_accounting", "as2d_session_run",
-            "as2d_budget_select")
+            "as2d_budget_select", "as2d_prefill")
 KERNEL_CLASSES = {"qkv": 0, "attention": 1, "o": 2, "gate_up": 3, "down": 4,
                   "lm_head": 5, "other": 6, "pass": 7}
 
@@ -138,6 +138,8 @@ _lib.as2d_session_run.argtypes = [ctypes.POINTER(as2d_session_spec), _P,
 _lib.as2d_session_run.restype = _S
 _lib.as2d_budget_select.argtypes = [_P, _P, _P, _P, _P, _S, _S, _S, _S, _P, _P, _P]
 _lib.as2d_budget_select.restype = _S
+_lib.as2d_prefill.argtypes = [_P, _P, _S, _P, _P]
+_lib.as2d_prefill.restype = _S
 _lib.as2d_last_error.argtypes = []
 _lib.as2d_last_error.restype = ctypes.c_char_p
 
@@ -477,6 +479,12 @@ class State:
             self.handle, [x.handle for x in bufs], b, self.batch, stream)
         _check(st, "as2d_verify_from_buffers")
         return k_used, rows
+
+    def prefill(self, tokens, first_token=None, stream=0):
+        """as2d_prefill: tokens and first_token are device int32 tensors."""
+        _check(_lib.as2d_prefill(self.handle, tokens.data_ptr(), tokens.numel(),
+                                 first_token.data_ptr() if first_token is not None else None,
+                                 stream), "as2d_prefill")
 
     def rollback(self, new_len, new_root, stream=0):
         _check(as2d_kv_rollback(self.handle, new_len, new_root, stream), "as2d_kv_rollback")

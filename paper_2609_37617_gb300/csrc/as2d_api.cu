@@ -339,6 +339,7 @@ extern "C" void as2d_kv_free(as2d_kv* kh) {
   cudaFree(kh->s.work);
   cudaFree(kh->s.rope_full);
   cudaFree(kh->s.cb_dev);
+  cudaFree(kh->s.pf_out);
   cudaFreeHost(kh->s.cb_host);
   delete kh;
 }
@@ -448,8 +449,12 @@ cudaError_t tc_project(int epi, const Model& m, KvState& s, const RowMap& rm, co
   return cudaSuccess;
 }
 
+// One verification pass.  force: keep every row whatever the greedy tokens
+// (prefill); root_override: device int32 [batch], the tokens forwarded in
+// place of the pending roots.
 as2d_status run_block(KvState& s, const int32_t* cand, const int32_t* k,
-                      const as2d_verify_out* out, cudaStream_t st) {
+                      const as2d_verify_out* out, cudaStream_t st, bool force = false,
+                      const int32_t* root_override = nullptr) {
   if (!out || !out->n_accepted || !out->correction_token)
     return fail(AS2D_ERR_INVALID_ARG, "out, out->n_accepted and out->correction_token are required");
   RowMap rm;
@@ -476,12 +481,12 @@ as2d_status run_block(KvState& s, const int32_t* cand, const int32_t* k,
   // sequence of kernels chained by programmatic dependent launch.  With
   // AS2D_PERSISTENT=1 in the environment, calls of at most 32 rows run it as
   // one persistent kernel instead (same arithmetic, same results).
-  if (mk_usable(s, rm.rows)) {
+  if (!force && !root_override && mk_usable(s, rm.rows)) {
     LAUNCH(AS2D_KERNEL_PASS, launch_mk(rm, m, s, cand, *out, st));
     for (int b = 0; b < s.batch; ++b) s.len_upper[b] += (k ? k[b] : 0) + 1;
     return AS2D_OK;
   }
-  LAUNCH(AS2D_KERNEL_OTHER, launch_embed(rm, m, s, cand, st));
+  LAUNCH(AS2D_KERNEL_OTHER, launch_embed(rm, m, s, cand, st, root_override));
   TcParams tp{};
   tp.h = s.h;
   tp.u = s.u;
@@ -516,12 +521,43 @@ as2d_status run_block(KvState& s, const int32_t* cand, const int32_t* k,
     LAUNCH(AS2D_KERNEL_DOWN, tc_project(TC_RESID, m, s, rm, m.w_down[l], s.tm_u, H, F, tp, st));
   }
   LAUNCH(AS2D_KERNEL_LM_HEAD, tc_project(TC_LOGITS, m, s, rm, m.lm_head, s.tm_xn, c.vocab, H, tp, st));
-  LAUNCH(AS2D_KERNEL_OTHER, launch_accept(rm, m, s, cand, *out, st));
+  LAUNCH(AS2D_KERNEL_OTHER, launch_accept(rm, m, s, cand, *out, st, force));
   for (int b = 0; b < s.batch; ++b) s.len_upper[b] += (k ? k[b] : 0) + 1;
   return AS2D_OK;
 }
 
 }  // namespace
+
+extern "C" as2d_status as2d_prefill(as2d_kv* kh, const int32_t* tokens, int32_t n,
+                                    int32_t* first_token, void* stream) {
+  g_err.clear();
+  if (!kh || !tokens || n < 1) return fail(AS2D_ERR_INVALID_ARG, "kv, tokens and n >= 1 are required");
+  KvState& s = kh->s;
+  if (s.batch != 1) return fail(AS2D_ERR_UNSUPPORTED, "prefill runs batch-1 states");
+  if (s.len_upper[0] + n > s.capacity)
+    return fail(AS2D_ERR_CAPACITY, "length bound + n exceeds the cache capacity");
+  if (!s.pf_out) {
+    const cudaError_t e = cudaMalloc(&s.pf_out, 2 * sizeof(int32_t));
+    if (e != cudaSuccess) {
+      s.pf_out = nullptr;
+      return fail(AS2D_ERR_CUDA, std::string("cudaMalloc: ") + cudaGetErrorString(e));
+    }
+  }
+  // chunks of at most AS2D_MAX_K + 1 tokens: the chunk's first token stands
+  // in for the pending root, the rest are kept as accepted candidates, and
+  // the greedy token after the chunk's last row becomes the root
+  for (int s0 = 0; s0 < n; s0 += kMaxK + 1) {
+    const int rows = (n - s0) < (kMaxK + 1) ? (n - s0) : (kMaxK + 1);
+    const int32_t k = rows - 1;
+    const bool last = s0 + rows == n;
+    const as2d_verify_out out{s.pf_out, (last && first_token) ? first_token : s.pf_out + 1,
+                              nullptr, nullptr};
+    const as2d_status rc = run_block(s, tokens + s0 + 1, &k, &out, (cudaStream_t)stream,
+                                     /*force=*/true, /*root_override=*/tokens + s0);
+    if (rc != AS2D_OK) return rc;
+  }
+  return AS2D_OK;
+}
 
 extern "C" as2d_status as2d_verify_block(as2d_kv* kh, const int32_t* candidates,
                                          const int32_t* k,

@@ -187,6 +187,7 @@ struct KvState {
   // candidates [batch][kMaxK], then n_accepted [batch] and correction [batch]
   int32_t* cb_dev = nullptr;
   int32_t* cb_host = nullptr;            // pinned, same layout
+  int32_t* pf_out = nullptr;             // [2] n_accepted, root of as2d_prefill chunks
 };
 
 // Error reporting shared by the translation units of the C-ABI: records the
@@ -196,10 +197,11 @@ void clear_error();
 
 // Launchers (k_basic.cu).  All enqueue on `st` and return cudaGetLastError().
 cudaError_t launch_embed(const RowMap& m, const Model& md, KvState& kv,
-                         const int32_t* cand, cudaStream_t st);
+                         const int32_t* cand, cudaStream_t st,
+                         const int32_t* root_override = nullptr);
 cudaError_t launch_accept(const RowMap& m, const Model& md, KvState& kv,
                           const int32_t* cand, const as2d_verify_out& out,
-                          cudaStream_t st);
+                          cudaStream_t st, bool force = false);
 cudaError_t launch_rollback(KvState& kv, const int32_t* new_len,
                             const int32_t* new_root, cudaStream_t st);
 // Fills kv.rope_full for positions [0, capacity).

@@ -35,7 +35,7 @@ __global__ void rope_table_kernel(float2* __restrict__ out, int d, double theta)
 // every position when there is one (rope_full), else computed.
 __global__ void __launch_bounds__(128) embed_kernel(
     RowMap m, const int32_t* __restrict__ cand, const int32_t* __restrict__ root,
-    const bf16* __restrict__ E, int H, int V, float* __restrict__ h, int32_t* err, int32_t* bad,
+    const int32_t* __restrict__ root_override, const bf16* __restrict__ E, int H, int V, float* __restrict__ h, int32_t* err, int32_t* bad,
     const int32_t* __restrict__ len, float2* __restrict__ rope, const float2* __restrict__ rope_full,
     int d, double theta, const float* __restrict__ g0, bf16* __restrict__ xn,
     float* __restrict__ ss, int ss_ld) {
@@ -50,7 +50,7 @@ __global__ void __launch_bounds__(128) embed_kernel(
     rope[(size_t)r * (d / 2) + e] =
         rope_full ? rope_full[(size_t)pos * (d / 2) + e] : rope_angle(pos, e, d, theta);
   }
-  int tok = (i == 0) ? root[b] : cand[m.start[b] - b + i - 1];
+  int tok = (i == 0) ? (root_override ? root_override[b] : root[b]) : cand[m.start[b] - b + i - 1];
   if (tok < 0 || tok >= V) {
     if (threadIdx.x == 0) {
       atomicOr(err, kErrBadToken);
@@ -102,10 +102,10 @@ __global__ void f32_from_bf16_kernel(float* dst, const bf16* src, int64_t n) {
 // ---- launchers ------------------------------------------------------------------------
 
 cudaError_t launch_embed(const RowMap& m, const Model& md, KvState& kv,
-                         const int32_t* cand, cudaStream_t st) {
+                         const int32_t* cand, cudaStream_t st, const int32_t* root_override) {
   ++kv.launches;
   return launch_pdl(embed_kernel, dim3(m.rows), dim3(128), 0, st, m, cand,
-                    (const int32_t*)kv.d_root, (const bf16*)md.embed, md.cfg.hidden,
+                    (const int32_t*)kv.d_root, root_override, (const bf16*)md.embed, md.cfg.hidden,
                     md.cfg.vocab, kv.h, kv.d_err, kv.d_err + 1, (const int32_t*)kv.d_len,
                     kv.rope, (const float2*)kv.rope_full, md.cfg.head_dim,
                     (double)md.cfg.rope_theta, md.attn_norm[0], kv.xn, kv.ss, kv.rows_alloc);
@@ -119,11 +119,11 @@ cudaError_t launch_rope_table(const Model& md, KvState& kv, cudaStream_t st) {
 
 cudaError_t launch_accept(const RowMap& m, const Model& md, KvState& kv,
                           const int32_t* cand, const as2d_verify_out& out,
-                          cudaStream_t st) {
+                          cudaStream_t st, bool force) {
   (void)md;
   ++kv.launches;
   AcceptArgs a{m, cand, kv.best, kv.d_len, kv.d_root, kv.d_err + 1, out.n_accepted,
-               out.correction_token, out.greedy};
+               out.correction_token, out.greedy, force ? 1 : 0};
   return launch_pdl(accept_kernel, dim3(m.batch), dim3(32), 0, st, a);
 }
 

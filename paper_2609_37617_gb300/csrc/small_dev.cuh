@@ -56,6 +56,7 @@ struct AcceptArgs {
   int32_t* n_out;
   int32_t* corr_out;
   int32_t* greedy_out;
+  int32_t force;  // 1: every row is kept whatever the greedy tokens (prefill)
 };
 
 // Accept scan of request b by one warp (App. C.2): g_i from the packed maxima,
@@ -74,7 +75,7 @@ __device__ __forceinline__ void accept_request(const AcceptArgs& a, int b, int l
   }
   const bool match = (lane < k) && (a.cand[r0 - b + lane] == g);
   const unsigned mm = __ballot_sync(0xFFFFFFFFu, match);
-  const int n = __ffs(~mm) - 1;  // bit k of mm is clear, so n <= k
+  const int n = a.force ? k : __ffs(~mm) - 1;  // bit k of mm is clear, so n <= k
   const int corr = __shfl_sync(0xFFFFFFFFu, g, n);
   if (lane == 0) {
     if (a.bad[b]) {

@@ -63,6 +63,7 @@ LAYER_KINDS = ("attn_norm", "w_q", "w_k", "w_v", "w_o", "mlp_norm",
                "w_gate", "w_up", "w_down")
 GAINS = ("attn_norm", "mlp_norm")
 S_ROOT = 0x20000000
+S_INSTR = 0x20000001
 
 
 def layer_stream(layer, kind):
@@ -149,6 +150,12 @@ def host_kv_request(cfg, req, kv_len, capacity, seed=0, poison=True):
         ks.append(pair[0])
         vs.append(pair[1])
     return ks, vs
+
+
+def instruction_tokens(cfg, n, seed=0):
+    """n instruction-suffix token ids, uniform over the vocabulary (the text
+    that follows the retained audio positions in the prompt)."""
+    return synth.uniform_int(n, seed, S_INSTR, cfg.vocab)
 
 
 def root_tokens(cfg, batch, seed=0):
