@@ -70,6 +70,9 @@ def parse():
     ap.add_argument("--drafter-kv-len", type=int, default=814)
     ap.add_argument("--session-tokens", type=int, default=256)
     ap.add_argument("--session-b", type=int, default=8)
+    ap.add_argument("--drafter-sms", type=int, default=0,
+                    help="--session: confine the drafter's grids to this many SMs and the "
+                         "target's to the rest (0: both use every SM)")
     ap.add_argument("--session-noise", type=float, default=0.25,
                     help="per-token substitution probability of the producer's text")
     return ap.parse_args()
@@ -666,6 +669,10 @@ def run_session(args, ws, rank, local):
         models.append(lib.Model(c, D.weight_pointers(c, w)))
         del w
         torch.cuda.empty_cache()
+    if args.drafter_sms > 0:
+        n_sm = torch.cuda.get_device_properties(local).multi_processor_count
+        models[0].set_sm_budget(n_sm - args.drafter_sms)
+        models[1].set_sm_budget(args.drafter_sms)
     cap_t = L0 + 2 * N + 64
     cap_d = DL0 + n_script + 16
     kc, vc = D.device_kv(cfg, [L0], cap_t, seed, poison=False)
@@ -723,7 +730,9 @@ def run_session(args, ws, rank, local):
                 "own decode steps for their cost)",
         "config": {"workload": f"{args.model} target (L0={L0}) + {args.drafter} drafter "
                                f"(L0={DL0}), N={N} committed tokens, b={b}, 8-token batches, "
-                               f"substitution p={args.session_noise}, 2% insertions, 2% deletions",
+                               f"substitution p={args.session_noise}, 2% insertions, 2% deletions"
+                               + (f", drafter on {args.drafter_sms} SMs and target on the rest"
+                                  if args.drafter_sms > 0 else ", both on every SM"),
                    "l2": "inputs larger than L2 (weights streamed per call)"},
         "runs": runs,
         "speedup_overlapped_vs_serial": round(s["T"] / a["T"], 4),

@@ -109,6 +109,16 @@ typedef struct as2d_verify_out {
 as2d_status as2d_model_load(const as2d_config* cfg, const as2d_weights* w,
                             as2d_model** out);
 
+/* Size this model's kernel grids for n_sms SMs (1 .. the device's count; the
+   default is the device's count), so that the pass can share the GPU with
+   other work confined to the remaining SMs -- for example a drafter on its
+   own stream (as2d_session_run).  The work split depends on (shape, n_sms)
+   only: results stay batch invariant and bit-identical for a given budget;
+   another budget adds partial sums in another order.  States created before
+   a larger budget was set refuse to run (AS2D_ERR_INVALID_ARG): set the
+   budget before as2d_kv_init_prefilled. */
+as2d_status as2d_model_set_sm_budget(as2d_model* model, int32_t n_sms);
+
 /* Bind a verification state of `batch` requests to a caller-allocated cache
    and its prefilled prefix (App. A.1: the retained audio KV plus the
    instruction, a valid prefix of the reference prompt).

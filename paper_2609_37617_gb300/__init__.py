@@ -39,7 +39,7 @@ EXPORTED = ("as2d_model_load", "as2d_kv_init_prefilled", "as2d_verify_block",
             "as2d_cbuf_publish", "as2d_cbuf_candidates", "as2d_cbuf_after_call",
             "as2d_cbuf_state", "as2d_cbuf_source_of", "as2d_cbuf_free",
             "as2d_verify_from_buffers", "as2d_interval_accounting", "as2d_session_run",
-            "as2d_budget_select", "as2d_prefill")
+            "as2d_budget_select", "as2d_prefill", "as2d_model_set_sm_budget")
 KERNEL_CLASSES = {"qkv": 0, "attention": 1, "o": 2, "gate_up": 3, "down": 4,
                   "lm_head": 5, "other": 6, "pass": 7}
 
@@ -138,6 +138,8 @@ _lib.as2d_session_run.argtypes = [ctypes.POINTER(as2d_session_spec), _P,
 _lib.as2d_session_run.restype = _S
 _lib.as2d_budget_select.argtypes = [_P, _P, _P, _P, _P, _S, _S, _S, _S, _P, _P, _P]
 _lib.as2d_budget_select.restype = _S
+_lib.as2d_model_set_sm_budget.argtypes = [_P, _S]
+_lib.as2d_model_set_sm_budget.restype = _S
 _lib.as2d_prefill.argtypes = [_P, _P, _S, _P, _P]
 _lib.as2d_prefill.restype = _S
 _lib.as2d_last_error.argtypes = []
@@ -384,6 +386,9 @@ class Model:
         st, h = as2d_model_load(self.cfg, pointers, shape.n_layers)
         _check(st, "as2d_model_load")
         self.handle = h
+
+    def set_sm_budget(self, n_sms):
+        _check(_lib.as2d_model_set_sm_budget(self.handle, int(n_sms)), "as2d_model_set_sm_budget")
 
     def close(self):
         if self.handle:

@@ -129,6 +129,7 @@ extern "C" as2d_status as2d_model_load(const as2d_config* cfg,
   int dev = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&m.sm_count, cudaDevAttrMultiProcessorCount, dev);
+  m.device_sm_count = m.sm_count;
   (void)d;
 
   const size_t qkv_packed = packed_elems(m.qkv_rows, (int)H);
@@ -215,6 +216,15 @@ extern "C" as2d_status as2d_model_load(const as2d_config* cfg,
   return AS2D_OK;
 }
 
+extern "C" as2d_status as2d_model_set_sm_budget(as2d_model* mh, int32_t n_sms) {
+  g_err.clear();
+  if (!mh) return fail(AS2D_ERR_INVALID_ARG, "model is NULL");
+  if (n_sms < 1 || n_sms > mh->m.device_sm_count)
+    return fail(AS2D_ERR_INVALID_ARG, "n_sms must be in [1, the device's SM count]");
+  mh->m.sm_count = n_sms;
+  return AS2D_OK;
+}
+
 extern "C" void as2d_model_free(as2d_model* mh) {
   if (!mh) return;
   cudaFree(mh->m.arena);
@@ -288,6 +298,7 @@ extern "C" as2d_status as2d_kv_init_prefilled(as2d_model* mh, int32_t batch,
   s.rope = cv.take<float2>(R * (m.cfg.head_dim / 2));
   s.ss = cv.take<float>(R * (H / 128));
   s.ws = cv.take<float>((size_t)m.sm_count * 2 * s.nb_max * 128);
+  s.ws_sms = m.sm_count;
   s.counters = cv.take<int>(max_tiles);
   s.n_counters = (int)max_tiles;
   s.qkv_part = cv.take<float>(qkv_tiles * s.qkv_split * R * 128);
@@ -473,6 +484,8 @@ as2d_status run_block(KvState& s, const int32_t* cand, const int32_t* k,
   rm.rows = rm.start[s.batch];
   if (total_k > 0 && !cand) return fail(AS2D_ERR_INVALID_ARG, "candidates is NULL");
   const Model& m = *s.model;
+  if (m.sm_count > s.ws_sms)
+    return fail(AS2D_ERR_INVALID_ARG, "the model's SM budget grew after this state was created");
   const as2d_config& c = m.cfg;
 
   // One pass of the verification step (Section 3.2; App. C.2): embedding

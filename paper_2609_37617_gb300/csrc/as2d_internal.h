@@ -111,7 +111,8 @@ struct Model {
   int qkv_rows;      // (n_q + 2 n_kv) * head_dim
   int q_dim;         // n_q * head_dim
   int kv_dim;        // n_kv * head_dim
-  int sm_count;
+  int sm_count;      // SMs the grids are sized for (the device's, or a budget)
+  int device_sm_count;
   void* arena = nullptr;  // every weight below lives here
   size_t arena_bytes = 0;
   const bf16* embed = nullptr;    // [V][H]
@@ -159,7 +160,8 @@ struct KvState {
   float2* rope_full = nullptr;  // [capacity][d/2] (cos, sin) of every position (own allocation)
   int rows_alloc = 0;        // activation rows allocated (>= every NB used)
   int nb_max = 16;
-  float* ws = nullptr;       // [sm_count][2][nb_max][128] partial GEMM tiles
+  float* ws = nullptr;       // [ws_sms][2][nb_max][128] partial GEMM tiles
+  int ws_sms = 0;            // the model's SM budget when ws was sized
   float* qkv_part = nullptr;   // [qkv tiles][qkv_split][rows_alloc][128] split-K sums
   float* qkv_rinv = nullptr;   // [rows_alloc] 1 / rms of each row at the QKV projection
   int qkv_split = 1;

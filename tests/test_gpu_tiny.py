@@ -197,3 +197,36 @@ def test_argument_and_device_errors(pair):
     with pytest.raises(lib.AS2DError):
         st.check()
     st.close()
+
+
+def test_reduced_sm_budget_keeps_parity(pair):
+    """A model whose grids are sized for 16 SMs (as2d_model_set_sm_budget)
+    still matches the oracle and stays batch invariant; a budget that grows
+    after a state was sized is refused."""
+    import torch
+    import paper_2609_37617_gb300 as lib
+    from synth import device as D
+    cfg = pair.cfg
+    dw = D.device_weights(cfg, 0)
+    torch.cuda.synchronize()
+    model = lib.Model(cfg, D.weight_pointers(cfg, dw))
+    del dw
+    with pytest.raises(lib.AS2DError):
+        model.set_sm_budget(0)
+    model.set_sm_budget(16)
+    root, oc, cont, cand = _workload_block(pair)
+    ores = pair.oracle.verify_block(oc, L0, root, cand)
+    kc, vc = D.device_kv(cfg, [L0], CAP, 0)
+    st = lib.State(model, [L0], CAP, kc, vc, [root])
+    n, corr, greedy, logits = run_gpu_block(st, cfg, [cand])
+    compare_block(ores, logits[:5], greedy[:5], n[0], corr[0], 4)
+    # the same row alone (k = 0 after a rollback) gives bitwise the same logits
+    st.rollback([L0], [root])
+    n0, c0, g0, lg0 = run_gpu_block(st, cfg, [[]])
+    assert np.array_equal(lg0[0], logits[0])
+    model.set_sm_budget(torch.cuda.get_device_properties(0).multi_processor_count)
+    with pytest.raises(lib.AS2DError):
+        run_gpu_block(st, cfg, [[]])
+    st.close()
+    model.close()
+
