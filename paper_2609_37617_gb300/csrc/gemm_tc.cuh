@@ -614,7 +614,7 @@ __global__ void __launch_bounds__(192, 1)
         ptx::tc_fence_before();
         __syncwarp();
         if (lane == 0) ptx::mbar_arrive(&acc_empty[buf]);
-        if (p.defer) {  // finished by tc_reduce_kernel, launched next
+        if (p.defer) {  // finished by tc_resid_finish_kernel, launched next
           u = send;
           continue;
         }
@@ -644,27 +644,6 @@ __global__ void __launch_bounds__(192, 1)
     ptx::tc_fence_after();
     ptx::tmem_dealloc(tmem, Sh::TMEM_COLS);
   }
-}
-
-// Finishes the tiles a stream-K launch left split between CTAs (p.defer):
-// one CTA of 128 threads per tile; the parts, the epilogue's operands and
-// the row prologue's loads are issued together (tc_reduce_tile).
-template <int NB, int EPI>
-__global__ void __launch_bounds__(128) tc_reduce_kernel(const __grid_constant__ TcParams p) {
-  using Sh = TcShape<NB>;
-  constexpr int SP = Sh::SP;
-  __shared__ float sC[128 * SP];
-  __shared__ float s_rinv[NB];
-  __shared__ float red[64];
-  __shared__ int s_pos[NB], s_req[NB];
-  const int tile = blockIdx.x;
-  const long long tstart = (long long)tile * p.kb, tend = tstart + p.kb;
-  const int c_first = tc_owner(tstart, p), c_last = tc_owner(tend - 1, p);
-  ptx::griddep_wait();
-  ptx::griddep_launch_dependents();
-  if (c_last == c_first) return;  // a whole tile, finished by its GEMM CTA
-  tc_reduce_tile<NB, EPI, 8, true>(p, sC, s_rinv, red, s_pos, s_req, tile, c_first,
-                                   c_last - c_first + 1, threadIdx.x, threadIdx.x);
 }
 
 // The residual epilogue of a stream-K launch's split tiles, one CTA of 128
@@ -725,9 +704,9 @@ cudaError_t tc_gemm_launch(const CUtensorMap& x, const TcParams& p, cudaStream_t
   if (attr != cudaSuccess) return attr;
   cudaError_t e = launch_pdl(tc_gemm_kernel<NB, EPI>, dim3(p.grid), dim3(192), smem, st, x, p);
   if (e != cudaSuccess || !p.defer || p.grid < 2) return e;
-  if (EPI == TC_RESID)
-    return launch_pdl(tc_resid_finish_kernel<NB>, dim3(p.n_tiles, p.rows), dim3(128), 0, st, p);
-  return launch_pdl(tc_reduce_kernel<NB, EPI>, dim3(p.n_tiles), dim3(128), 0, st, p);
+  // only the residual projections leave their split tiles to a finishing kernel
+  if (EPI != TC_RESID) return cudaErrorInvalidValue;
+  return launch_pdl(tc_resid_finish_kernel<NB>, dim3(p.n_tiles, p.rows), dim3(128), 0, st, p);
 }
 
 template <int EPI>
