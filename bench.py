@@ -475,7 +475,7 @@ def measure_prefill(args, lib, W, state, cfg, L0, root0, sh, stream, n_instr=64,
     ms = float(np.mean(times))
     return {"tokens": n_instr, "audio_positions": audio, "ms": round(ms, 3),
             "tok_s": round(n_instr / (ms / 1e3), 1),
-            "calls": -(-n_instr // 17), "reps": reps}
+            "passes": -(-n_instr // 64), "reps": reps}
 
 
 def select_budget(args, lib, state, traj, sweep, cfg, L0, root0, sh):

@@ -153,8 +153,11 @@ as2d_status as2d_verify_block(as2d_kv* kv, const int32_t* candidates,
 /* Instruction-suffix prefill (App. A.1: processing the instruction with the
    retained, compatible audio KV gives the initial decoding state): forwards
    tokens[0..n) (device int32 [n], ids in [0, vocab)) at positions
-   L .. L + n - 1 of a batch-1 state and keeps every entry, in chunks of at
-   most AS2D_MAX_K + 1 rows through the verification pass.  The pending root
+   L .. L + n - 1 of a batch-1 state and keeps every entry, in passes of up
+   to 64 rows through the verification pass (the first call allocates a
+   working state for such passes, kept until as2d_kv_free; its attention
+   buffers grow with the capacity, about 0.9 MB per 64 positions for the
+   7B shape).  The pending root
    before the call is discarded; afterwards L' = L + n and the root is the
    greedy token after tokens[n - 1] -- the first token of the response --
    also written to first_token (device int32 [1]) unless it is NULL.

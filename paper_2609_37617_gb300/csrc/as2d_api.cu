@@ -231,36 +231,15 @@ extern "C" void as2d_model_free(as2d_model* mh) {
   delete mh;
 }
 
-extern "C" as2d_status as2d_kv_init_prefilled(as2d_model* mh, int32_t batch,
-                                              const int32_t* kv_len,
-                                              int32_t capacity, void* k_cache,
-                                              void* v_cache,
-                                              const int32_t* root_tokens,
-                                              as2d_kv** out) {
-  g_err.clear();
-  if (!mh || !kv_len || !k_cache || !v_cache || !root_tokens || !out)
-    return fail(AS2D_ERR_INVALID_ARG, "a pointer argument is NULL");
-  if (batch < 1 || batch > kMaxBatch)
-    return fail(AS2D_ERR_INVALID_ARG, "batch must be in [1, AS2D_MAX_BATCH]");
-  if (capacity < 1) return fail(AS2D_ERR_INVALID_ARG, "capacity must be positive");
-  if (capacity > 65536)
-    return fail(AS2D_ERR_UNSUPPORTED, "capacity above 65536 positions is not supported");
-  const Model& m = mh->m;
-  for (int b = 0; b < batch; ++b) {
-    if (kv_len[b] < 0 || kv_len[b] >= capacity)
-      return fail(AS2D_ERR_CAPACITY, "kv_len must be in [0, capacity)");
-    if (root_tokens[b] < 0 || root_tokens[b] >= m.cfg.vocab)
-      return fail(AS2D_ERR_INVALID_ARG, "root token outside [0, vocab)");
-  }
-  as2d_kv* kh = new as2d_kv();
-  KvState& s = kh->s;
-  s.model = &mh->m;
-  s.batch = batch;
-  s.capacity = capacity;
-  s.k_cache = (bf16*)k_cache;
-  s.v_cache = (bf16*)v_cache;
-  s.len_upper.assign(kv_len, kv_len + batch);
-  s.max_rows = batch * (kMaxK + 1);
+namespace {
+
+// Sizes, allocates and carves the working memory of a state of `batch`
+// requests with up to `rows_per_request` rows each, and encodes the
+// activation descriptors.  Leaves s.work null on failure.
+as2d_status alloc_work(KvState& s, const Model& m, int batch, int capacity,
+                       int rows_per_request) {
+  s.max_k = rows_per_request - 1;
+  s.max_rows = batch * rows_per_request;
   s.nb_max = nb_for_rows(s.max_rows);
   s.rows_alloc = s.max_rows > s.nb_max ? s.max_rows : s.nb_max;
   const size_t R = s.rows_alloc, H = m.cfg.hidden, F = m.cfg.ffn;
@@ -276,12 +255,12 @@ extern "C" as2d_status as2d_kv_init_prefilled(as2d_model* mh, int32_t batch,
   bytes += align_up(qkv_tiles * s.qkv_split * R * 128 * 4, 256) + align_up(R * 4, 256);
   const int group = m.cfg.n_q_heads / m.cfg.n_kv_heads;
   s.attn_parts = attn_partitions(capacity);
-  s.attn_qmax = ((kMaxK + 1) * group + 15) / 16 * 16;
+  s.attn_qmax = (rows_per_request * group + 15) / 16 * 16;
   const size_t attn_rows = (size_t)batch * m.cfg.n_kv_heads * s.attn_parts * s.attn_qmax;
   bytes += align_up(attn_rows * m.cfg.head_dim * 4, 256) + align_up(attn_rows * 8, 256);
   cudaError_t e = cudaMalloc(&s.work, bytes);
   if (e != cudaSuccess) {
-    delete kh;
+    s.work = nullptr;
     return fail(AS2D_ERR_CUDA, std::string("cudaMalloc of the working memory: ") + cudaGetErrorString(e));
   }
   s.work_bytes = bytes;
@@ -315,9 +294,52 @@ extern "C" as2d_status as2d_kv_init_prefilled(as2d_model* mh, int32_t batch,
   }
   if (!ok) {
     cudaFree(s.work);
-    delete kh;
+    s.work = nullptr;
     return fail(AS2D_ERR_CUDA, "cuTensorMapEncodeTiled failed for an activation buffer");
   }
+  return AS2D_OK;
+}
+
+}  // namespace
+
+extern "C" as2d_status as2d_kv_init_prefilled(as2d_model* mh, int32_t batch,
+                                              const int32_t* kv_len,
+                                              int32_t capacity, void* k_cache,
+                                              void* v_cache,
+                                              const int32_t* root_tokens,
+                                              as2d_kv** out) {
+  g_err.clear();
+  if (!mh || !kv_len || !k_cache || !v_cache || !root_tokens || !out)
+    return fail(AS2D_ERR_INVALID_ARG, "a pointer argument is NULL");
+  if (batch < 1 || batch > kMaxBatch)
+    return fail(AS2D_ERR_INVALID_ARG, "batch must be in [1, AS2D_MAX_BATCH]");
+  if (capacity < 1) return fail(AS2D_ERR_INVALID_ARG, "capacity must be positive");
+  if (capacity > 65536)
+    return fail(AS2D_ERR_UNSUPPORTED, "capacity above 65536 positions is not supported");
+  const Model& m = mh->m;
+  for (int b = 0; b < batch; ++b) {
+    if (kv_len[b] < 0 || kv_len[b] >= capacity)
+      return fail(AS2D_ERR_CAPACITY, "kv_len must be in [0, capacity)");
+    if (root_tokens[b] < 0 || root_tokens[b] >= m.cfg.vocab)
+      return fail(AS2D_ERR_INVALID_ARG, "root token outside [0, vocab)");
+  }
+  as2d_kv* kh = new as2d_kv();
+  KvState& s = kh->s;
+  s.model = &mh->m;
+  s.batch = batch;
+  s.capacity = capacity;
+  s.k_cache = (bf16*)k_cache;
+  s.v_cache = (bf16*)v_cache;
+  s.len_upper.assign(kv_len, kv_len + batch);
+  {
+    const as2d_status rc = alloc_work(s, m, batch, capacity, kMaxK + 1);
+    if (rc != AS2D_OK) {
+      delete kh;
+      return rc;
+    }
+  }
+  cudaError_t e;
+  const size_t bytes = s.work_bytes;
   e = mk_prepare(m, s);
   if (e != cudaSuccess) {
     cudaFree(s.mk_mem);
@@ -351,6 +373,11 @@ extern "C" void as2d_kv_free(as2d_kv* kh) {
   cudaFree(kh->s.rope_full);
   cudaFree(kh->s.cb_dev);
   cudaFree(kh->s.pf_out);
+  if (kh->s.pf) {
+    // the prefill state's lengths, roots, flags and rotary table are this state's
+    cudaFree(kh->s.pf->work);
+    delete kh->s.pf;
+  }
   cudaFreeHost(kh->s.cb_host);
   delete kh;
 }
@@ -474,7 +501,7 @@ as2d_status run_block(KvState& s, const int32_t* cand, const int32_t* k,
   int total_k = 0;
   for (int b = 0; b < s.batch; ++b) {
     const int kb = k ? k[b] : 0;
-    if (kb < 0 || kb > kMaxK)
+    if (kb < 0 || kb > s.max_k)
       return fail(AS2D_ERR_INVALID_ARG, "k must be in [0, AS2D_MAX_K]");
     if (s.len_upper[b] + kb + 1 > s.capacity)
       return fail(AS2D_ERR_CAPACITY, "length bound + k + 1 exceeds the cache capacity");
@@ -556,20 +583,52 @@ extern "C" as2d_status as2d_prefill(as2d_kv* kh, const int32_t* tokens, int32_t 
       return fail(AS2D_ERR_CUDA, std::string("cudaMalloc: ") + cudaGetErrorString(e));
     }
   }
-  // chunks of at most AS2D_MAX_K + 1 tokens: the chunk's first token stands
-  // in for the pending root, the rest are kept as accepted candidates, and
-  // the greedy token after the chunk's last row becomes the root
-  for (int s0 = 0; s0 < n; s0 += kMaxK + 1) {
-    const int rows = (n - s0) < (kMaxK + 1) ? (n - s0) : (kMaxK + 1);
+  if (!s.pf) {
+    // a working state for passes of kPrefillRows rows over this state's cache
+    KvState* a = new KvState();
+    a->model = s.model;
+    a->batch = 1;
+    a->capacity = s.capacity;
+    a->k_cache = s.k_cache;
+    a->v_cache = s.v_cache;
+    a->len_upper = s.len_upper;
+    as2d_status rc = alloc_work(*a, *s.model, 1, s.capacity, kPrefillRows);
+    if (rc == AS2D_OK) {
+      const cudaError_t e = cudaMemset(a->work, 0, a->work_bytes);
+      if (e != cudaSuccess) {
+        cudaFree(a->work);
+        rc = fail(AS2D_ERR_CUDA, std::string("cudaMemset: ") + cudaGetErrorString(e));
+      }
+    }
+    if (rc != AS2D_OK) {
+      delete a;
+      return rc;
+    }
+    a->d_len = s.d_len;
+    a->d_root = s.d_root;
+    a->d_err = s.d_err;
+    a->rope_full = s.rope_full;
+    s.pf = a;
+  }
+  KvState& w = *s.pf;
+  w.len_upper = s.len_upper;
+  // passes of at most kPrefillRows tokens: the pass's first token stands in
+  // for the pending root, the rest are kept as accepted candidates, and the
+  // greedy token after the pass's last row becomes the root
+  as2d_status rc = AS2D_OK;
+  for (int s0 = 0; s0 < n && rc == AS2D_OK; s0 += kPrefillRows) {
+    const int rows = (n - s0) < kPrefillRows ? (n - s0) : kPrefillRows;
     const int32_t k = rows - 1;
     const bool last = s0 + rows == n;
     const as2d_verify_out out{s.pf_out, (last && first_token) ? first_token : s.pf_out + 1,
                               nullptr, nullptr};
-    const as2d_status rc = run_block(s, tokens + s0 + 1, &k, &out, (cudaStream_t)stream,
-                                     /*force=*/true, /*root_override=*/tokens + s0);
-    if (rc != AS2D_OK) return rc;
+    rc = run_block(w, tokens + s0 + 1, &k, &out, (cudaStream_t)stream,
+                   /*force=*/true, /*root_override=*/tokens + s0);
   }
-  return AS2D_OK;
+  s.len_upper = w.len_upper;
+  s.launches += w.launches;
+  w.launches = 0;
+  return rc;
 }
 
 extern "C" as2d_status as2d_verify_block(as2d_kv* kh, const int32_t* candidates,

@@ -17,6 +17,7 @@ namespace as2d {
 constexpr int kMaxBatch = AS2D_MAX_BATCH;
 constexpr int kMaxK = AS2D_MAX_K;
 constexpr int kMaxRows = kMaxBatch * (kMaxK + 1);
+constexpr int kPrefillRows = 64;  // token rows of one prefill pass
 
 typedef __nv_bfloat16 bf16;
 
@@ -145,7 +146,8 @@ struct KvState {
   int32_t* d_len = nullptr;   // [batch]
   int32_t* d_root = nullptr;  // [batch]
   int32_t* d_err = nullptr;   // [1]
-  // working memory, sized for batch * (kMaxK + 1) rows
+  // working memory, sized for batch * (max_k + 1) rows
+  int max_k = kMaxK;         // most candidates (rows - 1) of one request in a call
   int max_rows = 0;
   void* work = nullptr;
   size_t work_bytes = 0;
@@ -190,6 +192,10 @@ struct KvState {
   int32_t* cb_dev = nullptr;
   int32_t* cb_host = nullptr;            // pinned, same layout
   int32_t* pf_out = nullptr;             // [2] n_accepted, root of as2d_prefill chunks
+  // as2d_prefill's working state (batch 1, kPrefillRows rows per pass), made
+  // on first use; shares this state's cache, lengths, roots, error flags and
+  // rotary table
+  KvState* pf = nullptr;
 };
 
 // Error reporting shared by the translation units of the C-ABI: records the

@@ -66,6 +66,32 @@ __device__ __forceinline__ void accept_request(const AcceptArgs& a, int b, int l
   const RowMap& m = a.rm;
   const int r0 = m.start[b];
   const int k = m.start[b + 1] - r0 - 1;
+  if (a.force) {
+    // every row kept (prefill, up to kPrefillRows rows): the maxima cleared
+    // 32 rows at a time, the root is the greedy token after the last row
+    int g_last = 0;
+    for (int i = lane; i <= k; i += 32) {
+      const unsigned long long v = a.best[r0 + i];
+      const int g = (int)(0xFFFFFFFFu - (uint32_t)(v & 0xFFFFFFFFull));
+      a.best[r0 + i] = 0ull;
+      if (a.greedy_out) a.greedy_out[r0 + i] = g;
+      if (i == k) g_last = g;
+    }
+    g_last = __shfl_sync(0xFFFFFFFFu, g_last, k & 31);
+    if (lane == 0) {
+      if (a.bad[b]) {
+        a.n_out[b] = -1;
+        a.corr_out[b] = -1;
+        a.bad[b] = 0;
+      } else {
+        a.n_out[b] = k;
+        a.corr_out[b] = g_last;
+        a.len[b] += k + 1;
+        a.root[b] = g_last;
+      }
+    }
+    return;
+  }
   int g = 0;
   if (lane <= k) {
     const unsigned long long v = a.best[r0 + lane];
@@ -75,7 +101,7 @@ __device__ __forceinline__ void accept_request(const AcceptArgs& a, int b, int l
   }
   const bool match = (lane < k) && (a.cand[r0 - b + lane] == g);
   const unsigned mm = __ballot_sync(0xFFFFFFFFu, match);
-  const int n = a.force ? k : __ffs(~mm) - 1;  // bit k of mm is clear, so n <= k
+  const int n = __ffs(~mm) - 1;  // bit k of mm is clear, so n <= k
   const int corr = __shfl_sync(0xFFFFFFFFu, g, n);
   if (lane == 0) {
     if (a.bad[b]) {

@@ -69,18 +69,19 @@ def test_prefill_matches_oracle(pair):
     st.close()
 
 
-@pytest.mark.parametrize("chunks", [[1] * 20, [17, 3], [5, 15], [18, 2]])
+@pytest.mark.parametrize("chunks", [[1] * 100, [17, 83], [64, 36], [5, 90, 5], [99, 1]])
 def test_prefill_is_chunking_invariant(pair, chunks):
     """Any split of the suffix into prefill calls gives bitwise the same cache
-    and first token as one call (pathwise equivalence, batch invariance)."""
+    and first token as one call of 100 tokens (passes of 64 + 36 rows):
+    pathwise equivalence and batch invariance."""
     cfg = pair.cfg
-    instr = [int(t) for t in W.instruction_tokens(cfg, 20, 1)]
+    instr = [int(t) for t in W.instruction_tokens(cfg, 100, 1)]
     ref, first_ref = _prefill_gpu(pair, instr)
     st, first = _prefill_gpu(pair, instr, chunks)
     assert first == first_ref
     for l in range(cfg.n_layers):
-        assert np.array_equal(bf16_bits(st.kc[l, 0])[:, :L0 + 20], bf16_bits(ref.kc[l, 0])[:, :L0 + 20])
-        assert np.array_equal(bf16_bits(st.vc[l, 0])[:, :L0 + 20], bf16_bits(ref.vc[l, 0])[:, :L0 + 20])
+        assert np.array_equal(bf16_bits(st.kc[l, 0])[:, :L0 + 100], bf16_bits(ref.kc[l, 0])[:, :L0 + 100])
+        assert np.array_equal(bf16_bits(st.vc[l, 0])[:, :L0 + 100], bf16_bits(ref.vc[l, 0])[:, :L0 + 100])
     assert st.read_state() == ref.read_state()
     st.close()
     ref.close()
