@@ -24,6 +24,9 @@ def pair():
 
 @pytest.fixture(scope="module")
 def pair_gains():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no GPU")
     return Pair(W.TINY, seed=3, gains="random")
 
 
@@ -230,3 +233,39 @@ def test_reduced_sm_budget_keeps_parity(pair):
     st.close()
     model.close()
 
+
+
+def test_max_batch_max_k_and_capacity_edge(pair):
+    """AS2D_MAX_BATCH requests with AS2D_MAX_K candidates each (1088 rows, so
+    the projections run in several row chunks), ragged lengths, one request
+    ending exactly at the capacity: every request matches the oracle, and a
+    request verified alone gives bitwise the same rows."""
+    import paper_2609_37617_gb300 as lib
+    from synth import device as D
+    import torch
+    cfg = pair.cfg
+    B, K, cap = lib.AS2D_MAX_BATCH, lib.AS2D_MAX_K, CAP
+    lens = [cap - K - 1] + [16 + 3 * b for b in range(1, B)]
+    roots = [int(t) for t in W.root_tokens(cfg, B, 5)]
+    rng = np.random.default_rng(11)
+    cands = [[int(t) for t in rng.integers(0, cfg.vocab, K)] for _ in range(B)]
+    st = pair.state(lens, cap, roots)
+    n, corr, greedy, logits = run_gpu_block(st, cfg, cands)
+    ln, _ = st.read_state()
+    assert ln[0] <= cap
+    for b in (0, 1, 17, B - 1):
+        oc = pair.oracle_cache(lens[b], cap, req=b)
+        ores = pair.oracle.verify_block(oc, lens[b], roots[b], cands[b])
+        r0 = b * (K + 1)
+        compare_block(ores, logits[r0:r0 + K + 1], greedy[r0:r0 + K + 1], n[b], corr[b], K)
+    # request B-1 alone, on a copy of its cache
+    single = pair.state([lens[-1]], cap, [roots[-1]])
+    kc, vc = D.device_kv(cfg, lens, cap, pair.seed)
+    single.kc.copy_(kc[:, B - 1:B])
+    single.vc.copy_(vc[:, B - 1:B])
+    torch.cuda.synchronize()
+    n1, c1, g1, lg1 = run_gpu_block(single, cfg, [cands[-1]])
+    assert np.array_equal(lg1, logits[(B - 1) * (K + 1):])
+    st.check()
+    single.close()
+    st.close()
