@@ -70,6 +70,11 @@ def parse():
     ap.add_argument("--drafter-kv-len", type=int, default=814)
     ap.add_argument("--session-tokens", type=int, default=256)
     ap.add_argument("--session-b", type=int, default=8)
+    ap.add_argument("--cpu-drafter", action="store_true",
+                    help="--session: the producer runs the cpu-draft decoder on the host cores "
+                         "instead of a GPU drafter")
+    ap.add_argument("--cpu-threads", type=int, default=0,
+                    help="host threads of the CPU drafter (0: half the cores, at most 8)")
     ap.add_argument("--drafter-sms", type=int, default=0,
                     help="--session: confine the drafter's grids to this many SMs and the "
                          "target's to the rest (0: both use every SM)")
@@ -663,24 +668,41 @@ def run_session(args, ws, rank, local):
     s_d = torch.cuda.Stream(priority=0)
     models, states = [], []
     n_script = 2 * N + 64
+    cpu = None
+    if args.cpu_drafter:
+        ccfg = model_shape("cpu-draft")
+        hw = W.host_weights(ccfg, seed + 202)
+        f32 = lambda b: (np.asarray(b, dtype=np.uint16).astype(np.uint32) << 16).view(np.float32)
+        host = {k: f32(hw[k]) for k in ("embed", "final_norm", "lm_head")}
+        for name in ("attn_norm", "w_q", "w_k", "w_v", "w_o", "mlp_norm", "w_gate", "w_up", "w_down"):
+            host[name] = [f32(hw[f"{name}.{l}"]) for l in range(ccfg.n_layers)]
+        # half the host cores: more threads slow the verifier's own host thread
+        cpu_threads = args.cpu_threads or max(1, min(8, (os.cpu_count() or 8) // 2))
+        cpu = lib.CpuDecoder(ccfg, host, n_script + 16, cpu_threads, 1)
+        del host, hw
+        dcfg = None
     for c, L, sd in ((cfg, L0, seed), (dcfg, DL0, seed + 101)):
+        if c is None:
+            continue
         w = D.device_weights(c, sd)
         torch.cuda.synchronize()
         models.append(lib.Model(c, D.weight_pointers(c, w)))
         del w
         torch.cuda.empty_cache()
-    if args.drafter_sms > 0:
+    if args.drafter_sms > 0 and cpu is None:
         n_sm = torch.cuda.get_device_properties(local).multi_processor_count
         models[0].set_sm_budget(n_sm - args.drafter_sms)
         models[1].set_sm_budget(args.drafter_sms)
     cap_t = L0 + 2 * N + 64
     cap_d = DL0 + n_script + 16
     kc, vc = D.device_kv(cfg, [L0], cap_t, seed, poison=False)
-    dkc, dvc = D.device_kv(dcfg, [DL0], cap_d, seed + 101, poison=False)
     root_t = int(W.root_tokens(cfg, 1, seed)[0])
-    root_d = int(W.root_tokens(dcfg, 1, seed + 101)[0])
     target = lib.State(models[0], [L0], cap_t, kc, vc, [root_t])
-    drafter = lib.State(models[1], [DL0], cap_d, dkc, dvc, [root_d])
+    drafter = None
+    if cpu is None:
+        dkc, dvc = D.device_kv(dcfg, [DL0], cap_d, seed + 101, poison=False)
+        root_d = int(W.root_tokens(dcfg, 1, seed + 101)[0])
+        drafter = lib.State(models[1], [DL0], cap_d, dkc, dvc, [root_d])
 
     # the target's greedy text (untimed), then the producer's noisy copy
     nbuf = torch.zeros(1, dtype=torch.int32, device="cuda")
@@ -695,16 +717,21 @@ def run_session(args, ws, rank, local):
     def one(kind):
         target.rollback([L0], [root_t], s_t.cuda_stream)
         target.read_state(s_t.cuda_stream)
-        drafter.rollback([DL0], [root_d], s_d.cuda_stream)
-        drafter.read_state(s_d.cuda_stream)
+        if drafter is not None:
+            drafter.rollback([DL0], [root_d], s_d.cuda_stream)
+            drafter.read_state(s_d.cuda_stream)
+        else:
+            cpu.reset(0, 1)
         torch.cuda.synchronize()
         buf = lib.CandidateBuffer(8)
         sc = [] if kind == "target_only" else script
         comm, st = lib.session_run(target, drafter if sc else None, buf, sc, b, N,
                                    kind == "overlapped", target_stream=s_t.cuda_stream,
-                                   drafter_stream=s_d.cuda_stream)
+                                   drafter_stream=s_d.cuda_stream,
+                                   cpu_drafter=cpu if sc else None)
         target.check(s_t.cuda_stream)
-        drafter.check(s_d.cuda_stream)
+        if drafter is not None:
+            drafter.check(s_d.cuda_stream)
         m = min(len(comm), len(greedy_h))
         assert comm[:m] == greedy_h[:m], f"{kind}: committed text differs from greedy decoding"
         st["tok_s"] = st["committed"] / st["T"]
@@ -728,8 +755,10 @@ def run_session(args, ws, rank, local):
         "data": "synthetic (seeded random-init weights and KV; the producer publishes the "
                 "target's greedy text with seeded corruption while running the drafter's "
                 "own decode steps for their cost)",
-        "config": {"workload": f"{args.model} target (L0={L0}) + {args.drafter} drafter "
-                               f"(L0={DL0}), N={N} committed tokens, b={b}, 8-token batches, "
+        "config": {"workload": f"{args.model} target (L0={L0}) + "
+                               + (f"cpu-draft drafter on {cpu_threads} host threads"
+                                  if cpu is not None else f"{args.drafter} drafter (L0={DL0})")
+                               + f", N={N} committed tokens, b={b}, 8-token batches, "
                                f"substitution p={args.session_noise}, 2% insertions, 2% deletions"
                                + (f", drafter on {args.drafter_sms} SMs and target on the rest"
                                   if args.drafter_sms > 0 else ", both on every SM"),
@@ -743,7 +772,10 @@ def run_session(args, ws, rank, local):
     }
     print(json.dumps(line), flush=True)
     target.close()
-    drafter.close()
+    if drafter is not None:
+        drafter.close()
+    if cpu is not None:
+        cpu.close()
     for m in models:
         m.close()
 

@@ -356,6 +356,28 @@ as2d_status as2d_verify_from_buffers(as2d_kv* kv, as2d_cbuf* const* bufs, int32_
    Section 3.1: the producer runs without target feedback and the target
    never waits for it.) */
 
+/* A small decoder on the host cores: a producer placed on a different
+   processor than the target, as the paper places drafter and target on
+   different processors of one device.  fp32, one greedy decode step per
+   call over its own cache (positions 0, 1, ...), matrix-vector products
+   split over `threads` OpenMP threads.  w holds HOST float arrays in the
+   layouts of as2d_weights (per-layer members: host arrays of host pointers);
+   they are copied.  The shape rules of as2d_config do not apply (any
+   positive sizes, n_q % n_kv == 0, even head_dim). */
+typedef struct as2d_cpu_decoder as2d_cpu_decoder;
+as2d_status as2d_cpu_decoder_create(const as2d_config* cfg, const as2d_weights* w,
+                                    int32_t capacity, int32_t threads, int32_t root,
+                                    as2d_cpu_decoder** out);
+/* Forward the pending root at the next position, append its keys and values,
+   make the greedy token the new root and return it in *token_out (may be
+   NULL).  AS2D_ERR_CAPACITY when the cache is full. */
+as2d_status as2d_cpu_decoder_step(as2d_cpu_decoder* d, int32_t* token_out);
+/* The last step's logits: host float [vocab]. */
+as2d_status as2d_cpu_decoder_logits(as2d_cpu_decoder* d, float* logits);
+/* Back to an earlier length (<= the current one) with pending root `root`. */
+as2d_status as2d_cpu_decoder_reset(as2d_cpu_decoder* d, int32_t len, int32_t root);
+void as2d_cpu_decoder_free(as2d_cpu_decoder* d);
+
 /* Service-interval accounting over [0, T].  p: host double [np][2] producer
    service intervals (start, end); v: host double [nv][2] verifier
    intervals; each is clipped to [0, T] and merged with the overlapping
@@ -385,6 +407,8 @@ typedef struct as2d_session_spec {
                              waits, whenever fewer than b candidates are ready    */
   void* target_stream;
   void* drafter_stream;
+  as2d_cpu_decoder* cpu_drafter;  /* when not NULL (and drafter is NULL): one
+                                     host-core decode step per produced token */
 } as2d_session_spec;
 
 typedef struct as2d_session_stats {

@@ -39,7 +39,9 @@ EXPORTED = ("as2d_model_load", "as2d_kv_init_prefilled", "as2d_verify_block",
             "as2d_cbuf_publish", "as2d_cbuf_candidates", "as2d_cbuf_after_call",
             "as2d_cbuf_state", "as2d_cbuf_source_of", "as2d_cbuf_free",
             "as2d_verify_from_buffers", "as2d_interval_accounting", "as2d_session_run",
-            "as2d_budget_select", "as2d_prefill", "as2d_model_set_sm_budget")
+            "as2d_budget_select", "as2d_prefill", "as2d_model_set_sm_budget",
+            "as2d_cpu_decoder_create", "as2d_cpu_decoder_step", "as2d_cpu_decoder_logits",
+            "as2d_cpu_decoder_reset", "as2d_cpu_decoder_free")
 KERNEL_CLASSES = {"qkv": 0, "attention": 1, "o": 2, "gate_up": 3, "down": 4,
                   "lm_head": 5, "other": 6, "pass": 7}
 
@@ -76,7 +78,7 @@ class as2d_session_spec(ctypes.Structure):
                 ("n_script", ctypes.c_int32), ("b", ctypes.c_int32),
                 ("publish_every", ctypes.c_int32), ("n_commit", ctypes.c_int32),
                 ("overlapped", ctypes.c_int32), ("target_stream", ctypes.c_void_p),
-                ("drafter_stream", ctypes.c_void_p)]
+                ("drafter_stream", ctypes.c_void_p), ("cpu_drafter", ctypes.c_void_p)]
 
 
 class as2d_session_stats(ctypes.Structure):
@@ -142,6 +144,16 @@ _lib.as2d_model_set_sm_budget.argtypes = [_P, _S]
 _lib.as2d_model_set_sm_budget.restype = _S
 _lib.as2d_prefill.argtypes = [_P, _P, _S, _P, _P]
 _lib.as2d_prefill.restype = _S
+_lib.as2d_cpu_decoder_create.argtypes = [ctypes.POINTER(as2d_config), ctypes.POINTER(as2d_weights),
+                                         _S, _S, _S, ctypes.POINTER(ctypes.c_void_p)]
+_lib.as2d_cpu_decoder_step.argtypes = [_P, ctypes.POINTER(ctypes.c_int32)]
+_lib.as2d_cpu_decoder_logits.argtypes = [_P, _P]
+_lib.as2d_cpu_decoder_reset.argtypes = [_P, _S, _S]
+_lib.as2d_cpu_decoder_free.argtypes = [_P]
+_lib.as2d_cpu_decoder_free.restype = None
+for _n in ("as2d_cpu_decoder_create", "as2d_cpu_decoder_step", "as2d_cpu_decoder_logits",
+           "as2d_cpu_decoder_reset"):
+    getattr(_lib, _n).restype = _S
 _lib.as2d_last_error.argtypes = []
 _lib.as2d_last_error.restype = ctypes.c_char_p
 
@@ -333,15 +345,70 @@ def as2d_session_run(spec, n_commit, b):
     return st, list(comm[:max(stats.committed, 0)]), d
 
 
+class CpuDecoder:
+    """Owns an as2d_cpu_decoder built from host fp32 weights: `host` maps the
+    names of as2d_weights to float32 numpy arrays (per-layer names to lists)."""
+
+    def __init__(self, shape, host, capacity, threads, root):
+        import numpy as np
+        self._keep = {k: ([np.ascontiguousarray(a, dtype=np.float32) for a in v]
+                          if isinstance(v, list) else np.ascontiguousarray(v, dtype=np.float32))
+                      for k, v in host.items()}
+        w = as2d_weights()
+        for name in ("embed", "final_norm", "lm_head"):
+            setattr(w, name, self._keep[name].ctypes.data)
+        self._arrs = []
+        for name in ("attn_norm", "w_q", "w_k", "w_v", "w_o", "mlp_norm", "w_gate", "w_up",
+                     "w_down"):
+            arr = (ctypes.c_void_p * shape.n_layers)(*[a.ctypes.data for a in self._keep[name]])
+            self._arrs.append(arr)
+            setattr(w, name, ctypes.cast(arr, ctypes.c_void_p))
+        cfg = as2d_config(shape.n_layers, shape.hidden, shape.n_q, shape.n_kv, shape.head_dim,
+                          shape.ffn, shape.vocab, float(shape.rope_theta), float(shape.rms_eps))
+        h = ctypes.c_void_p()
+        _check(_lib.as2d_cpu_decoder_create(ctypes.byref(cfg), ctypes.byref(w), capacity, threads,
+                                            root, ctypes.byref(h)), "as2d_cpu_decoder_create")
+        self.handle = h.value
+        self.vocab = shape.vocab
+        self._keep = None  # copied by the library
+
+    def step(self):
+        t = ctypes.c_int32()
+        _check(_lib.as2d_cpu_decoder_step(self.handle, ctypes.byref(t)), "as2d_cpu_decoder_step")
+        return t.value
+
+    def logits(self):
+        import numpy as np
+        out = np.empty(self.vocab, dtype=np.float32)
+        _check(_lib.as2d_cpu_decoder_logits(self.handle, out.ctypes.data),
+               "as2d_cpu_decoder_logits")
+        return out
+
+    def reset(self, length, root):
+        _check(_lib.as2d_cpu_decoder_reset(self.handle, length, root), "as2d_cpu_decoder_reset")
+
+    def close(self):
+        if self.handle:
+            _lib.as2d_cpu_decoder_free(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
 def session_run(target, drafter, buf, script, b, n_commit, overlapped, publish_every=8,
-                target_stream=0, drafter_stream=0):
+                target_stream=0, drafter_stream=0, cpu_drafter=None):
     """Run a producer/verifier session (as2d_session_run) on State objects and
     a CandidateBuffer; returns (committed tokens, stats dict)."""
     arr = _i32_array(script) if len(script) else None
     spec = as2d_session_spec(target.handle, drafter.handle if drafter is not None else None,
                              buf.handle, ctypes.cast(arr, ctypes.c_void_p) if arr else None,
                              len(script), b, publish_every, n_commit, int(bool(overlapped)),
-                             target_stream, drafter_stream)
+                             target_stream, drafter_stream,
+                             cpu_drafter.handle if cpu_drafter is not None else None)
     st, comm, stats = as2d_session_run(spec, n_commit, b)
     _check(st, "as2d_session_run")
     return comm, stats

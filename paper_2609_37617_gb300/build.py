@@ -15,7 +15,7 @@ NVCC = os.path.join(CUDA_HOME, "bin", "nvcc")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 CFLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC",
           "-I", os.path.join(ROOT, "include"), "-I", os.path.join(HERE, "csrc"),
-          "--expt-relaxed-constexpr", "-Xptxas", "-warn-spills"]
+          "--expt-relaxed-constexpr", "-Xptxas", "-warn-spills", "-Xcompiler", "-fopenmp"]
 LIB = os.path.join(HERE, "libas2d.so")
 OBJ_DIR = os.path.join(HERE, "_build")
 
@@ -56,7 +56,7 @@ def build(force=False, verbose_ptxas=False):
     objs = [o for o, _ in results]
     tmp = LIB + ".tmp"
     r = subprocess.run([NVCC, *ARCH, "-shared", "-cudart", "shared",
-                        "-Xlinker", f"-rpath,{CUDA_HOME}/lib64", *objs, "-o", tmp],
+                        "-Xlinker", f"-rpath,{CUDA_HOME}/lib64", *objs, "-lgomp", "-o", tmp],
                        capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")

@@ -111,6 +111,12 @@ struct Producer {
   bool batch() {
     const double a = since(t0);
     const int n = std::min(sp.publish_every, sp.n_script - published);
+    if (sp.cpu_drafter && !sp.drafter) {
+      for (int i = 0; i < n; ++i) {
+        const as2d_status st = as2d_cpu_decoder_step(sp.cpu_drafter, nullptr);
+        if (st != AS2D_OK) return fail(st);
+      }
+    }
     if (sp.drafter) {
       for (int i = 0; i < n; ++i) {
         as2d_verify_out o{d_out + i, d_out + AS2D_CBUF_BATCH + i, nullptr, nullptr};

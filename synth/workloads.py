@@ -55,7 +55,10 @@ M1P5B = ModelConfig("1.5b", 28, 1536, 12, 2, 128, 8960, 151936)
 M7B = ModelConfig("7b", 28, 3584, 28, 4, 128, 18944, 152064)
 # 7B-shaped decoder with two layers: small enough for profiler captures
 M7B_2L = ModelConfig("7b-2l", 2, 3584, 28, 4, 128, 18944, 152064)
-MODELS = {m.name: m for m in (TINY, M1P5B, M7B, M7B_2L)}
+# a small drafter for the host cores (its own vocabulary: the producer's text
+# is re-tokenised for the target)
+CPU_DRAFT = ModelConfig("cpu-draft", 4, 512, 8, 2, 64, 1408, 8192)
+MODELS = {m.name: m for m in (TINY, M1P5B, M7B, M7B_2L, CPU_DRAFT)}
 
 # ---- stream ids ------------------------------------------------------------
 S_EMBED, S_LM_HEAD, S_FINAL_NORM = 1, 2, 3
