@@ -64,6 +64,8 @@ def parse():
                     help="block sizes k for the verify-time sweep ('' to skip); the budget "
                          "selection needs all of 0..16")
     ap.add_argument("--sweep-blocks", type=int, default=24)
+    ap.add_argument("--long-kv-len", type=int, default=15128,
+                    help="prefix length of the long-context sweep (0 to skip)")
     ap.add_argument("--session", action="store_true",
                     help="producer/verifier session line instead of the verify-step line")
     ap.add_argument("--drafter", default="1.5b", help="drafter model shape for --session")
@@ -374,6 +376,9 @@ def run_ours(args, ws, rank, local):
         if not args.no_e2e:
             e2e = run_e2e(args, lib, W, state, traj, plans, cfg, L0, root0, sh, stream)
         prefill = measure_prefill(args, lib, W, state, cfg, L0, root0, sh, stream)
+        long_ctx = None
+        if args.long_kv_len > 0 and args.model == "7b":
+            long_ctx = measure_long_context(args, lib, D, W, model, cfg, sh, stream, seed)
 
     if ws > 1:
         elapsed_ms, committed_all = reduce_ranks(elapsed_ms, committed, "cuda")
@@ -442,6 +447,7 @@ def run_ours(args, ws, rank, local):
         "k_sweep": sweep,
         "budget": budget,
         "prefill": prefill,
+        "long_context": long_ctx,
         "clocks": clk,
         "e2e": e2e,
     }
@@ -453,6 +459,51 @@ def run_ours(args, ws, rank, local):
     model.close()
     if ws > 1:
         dist.destroy_process_group()
+
+
+def measure_long_context(args, lib, D, W, model, cfg, sh, stream, seed, ks=(1, 4, 8, 16),
+                         blocks=16):
+    """Verify time at a long retained prefix (10 min of audio at 25 tokens/s
+    plus 128 instruction positions): `blocks` blocks per k from the same
+    prefix, uniform candidates (the time does not depend on acceptance), CUDA
+    events on the launching stream; the roofline counts the prefix's KV."""
+    import torch
+    L = args.long_kv_len
+    cap = L + (max(ks) + 1) * blocks + 64
+    kc, vc = D.device_kv(cfg, [L], cap, seed, poison=False)
+    st = lib.State(model, [L], cap, kc, vc, [1])
+    peak, _ = load_peaks()
+    rng = np.random.default_rng(seed + 77)
+    n = torch.zeros(1, dtype=torch.int32, device="cuda")
+    c = torch.zeros(1, dtype=torch.int32, device="cuda")
+    out = []
+    for k in ks:
+        cand = torch.from_numpy(rng.integers(0, cfg.vocab, (blocks, k)).astype(np.int32)).cuda()
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(blocks)]
+        st.rollback([L], [1], sh)
+        st.read_state(sh)
+        st.verify(cand[0], [k], n, c, stream=sh)          # warm-up
+        st.rollback([L], [1], sh)
+        st.read_state(sh)
+        torch.cuda.synchronize()
+        for i in range(blocks):
+            ev[i][0].record(stream)
+            st.verify(cand[i], [k], n, c, stream=sh)
+            ev[i][1].record(stream)
+        torch.cuda.synchronize()
+        us = float(np.mean([a.elapsed_time(b) * 1e3 for a, b in ev]))
+        ln, _ = st.read_state(sh)
+        mean_len = (L + ln[0]) / 2.0
+        bts = bytes_per_block(cfg, mean_len, k)
+        out.append({"k": k, "verify_us_mean": round(us, 1),
+                    "kv_bytes": int((mean_len + k + 1) * cfg.kv_bytes_per_pos()),
+                    "frac": round(bts / (peak * 1e9) / (us / 1e6), 4)})
+    st.check(sh)
+    st.close()
+    del kc, vc
+    torch.cuda.empty_cache()
+    return {"kv_len": L, "blocks_per_k": blocks, "sweep": out}
 
 
 def measure_prefill(args, lib, W, state, cfg, L0, root0, sh, stream, n_instr=64, reps=5):
