@@ -23,7 +23,8 @@
 // are fixed multiples of 64 positions, so a query's partial results do not
 // depend on the other rows of the call (batch invariance).
 // Pass 2 (attn_merge_kernel): per (row, query head) the partitions' (max,
-// sum, unnormalised output) are combined in partition order (log-sum-exp).
+// sum, unnormalised output) are combined (log-sum-exp) in an order fixed by
+// the row's own number of partitions.
 #include "attn_dev.cuh"
 
 namespace as2d {
@@ -72,13 +73,93 @@ __global__ void __launch_bounds__(D / 2) qkv_finish_kernel(AttnArgs a) {
   }
 }
 
+// Pass 2 for one (row, query head) per CTA of D x (1..4) threads.  All the
+// partitions' (max, sum) pairs are loaded together into shared memory; the
+// maximum, the weights 2^(m_p - M) and the total (warp 0: lane e adds
+// partitions e, e + 32, ... in order, then a butterfly) follow; the outputs
+// are added by gs = min(4, ceil(parts / 32)) groups of D threads, group q
+// taking a contiguous run of partitions in order, 32 loads in flight, and the
+// groups' sums are added in group order.  Every order depends on the row's
+// own number of partitions alone; with at most 32 partitions (positions below
+// 2048) it is the single in-order sum.
+constexpr int kMergeGroups = 4;
+
 template <int D>
-__global__ void __launch_bounds__(D) attn_merge_kernel(AttnArgs a) {
+__global__ void __launch_bounds__(kMergeGroups * D) attn_merge_kernel(AttnArgs a) {
+  constexpr int PF = 32;
+  __shared__ float2 s_ml[kMaxParts];
+  __shared__ float s_w[kMaxParts];
+  __shared__ float s_red[kMergeGroups * D / 32];
+  __shared__ float s_o[kMergeGroups - 1][D];
+  __shared__ float s_l;
   ptx::griddep_wait();
   ptx::griddep_launch_dependents();
-  __shared__ float w[kMaxParts];
-  __shared__ float s_l;
-  merge_item<D>(a, blockIdx.x, blockIdx.y, w, &s_l, threadIdx.x, blockDim.x, 0);
+  const int r = blockIdx.x, j = blockIdx.y, tid = threadIdx.x, nthr = blockDim.x;
+  const int G = a.nq / a.nkv;
+  const int b = row_request(a.rm, r);
+  const int i = r - a.rm.start[b];
+  const int g = j / G, qr = i * G + (j - g * G);
+  const int pos = a.len[b] + i;
+  const int nparts = pos / kPart + 1;
+  const size_t base = (size_t)(b * a.nkv + g) * a.parts_max * a.qmax + qr;
+  const int want = (nparts + 31) / 32;
+  const int gs = want < kMergeGroups ? want : kMergeGroups;
+  const int chunk = (nparts + gs - 1) / gs;
+  const int grp = tid / D, e = tid - grp * D;
+  const int p_begin = grp * chunk;
+  const int p_end = (p_begin + chunk) < nparts ? (p_begin + chunk) : nparts;
+  // the group's first PF outputs are in flight with the (max, sum) loads
+  float ov[PF];
+  if (grp < gs) {
+#pragma unroll
+    for (int u = 0; u < PF; ++u)
+      ov[u] = (p_begin + u < p_end) ? a.ws_o[(base + (size_t)(p_begin + u) * a.qmax) * D + e] : 0.f;
+  }
+  for (int p = tid; p < nparts; p += nthr) s_ml[p] = a.ws_ml[base + (size_t)p * a.qmax];
+  __syncthreads();
+  float M = -INFINITY;
+  for (int p = tid; p < nparts; p += nthr) M = fmaxf(M, s_ml[p].x);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xFFFFFFFFu, M, o));
+  if ((tid & 31) == 0) s_red[tid >> 5] = M;
+  __syncthreads();
+  M = s_red[0];
+  for (int w = 1; w < nthr / 32; ++w) M = fmaxf(M, s_red[w]);
+  for (int p = tid; p < nparts; p += nthr) {
+    const float mp = s_ml[p].x;
+    s_w[p] = (mp == -INFINITY) ? 0.f : exp2f(mp - M);
+  }
+  __syncthreads();
+  if (tid < 32) {
+    float l = 0.f;
+    for (int p = tid; p < nparts; p += 32) l += s_ml[p].y * s_w[p];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xFFFFFFFFu, l, o);
+    if (tid == 0) s_l = l;
+  }
+  float o = 0.f;
+  if (grp < gs) {
+    for (int p0 = p_begin; p0 < p_end; p0 += PF) {
+      if (p0 > p_begin) {
+#pragma unroll
+        for (int u = 0; u < PF; ++u)
+          ov[u] = (p0 + u < p_end) ? a.ws_o[(base + (size_t)(p0 + u) * a.qmax) * D + e] : 0.f;
+      }
+#pragma unroll
+      for (int u = 0; u < PF; ++u)
+        if (p0 + u < p_end) o += ov[u] * s_w[p0 + u];
+    }
+    if (grp > 0) s_o[grp - 1][e] = o;
+  }
+  __syncthreads();
+  if (grp == 0) {
+    for (int q = 1; q < gs; ++q) o += s_o[q - 1][e];
+    const float ov_ = o / s_l;
+    const bf16 oh = __float2bfloat16_rn(ov_);
+    a.ao[(size_t)r * a.nq * D + (size_t)j * D + e] = oh;
+    a.ao[(size_t)(a.lo_row + r) * a.nq * D + (size_t)j * D + e] =
+        __float2bfloat16_rn(ov_ - __bfloat162float(oh));
+  }
 }
 
 }  // namespace
@@ -120,6 +201,10 @@ cudaError_t launch_attention_split(const RowMap& m, const Model& md, KvState& kv
   a.qkv_split = kv.qkv_split;
   a.qkv_ld = kv.rows_alloc;
   const dim3 gf(m.rows, c.n_q_heads + 2 * c.n_kv_heads);
+  // merge groups for the call's longest row (each row uses min(4, its own
+  // partitions / 32 rounded up) of them)
+  int mg = (parts + 31) / 32;
+  mg = mg < 1 ? 1 : (mg > kMergeGroups ? kMergeGroups : mg);
   // Eight warps stage a partition fastest; when there are more items than
   // SMs, one warp per 16 query rows of the largest request (at least four,
   // for the staging copies) lets two CTAs share an SM, so long prefixes need
@@ -141,11 +226,11 @@ cudaError_t launch_attention_split(const RowMap& m, const Model& md, KvState& kv
   if (c.head_dim == 128) {
     e = launch_pdl(qkv_finish_kernel<128>, gf, dim3(64), 0, st, a);
     if (e == cudaSuccess) e = launch_pdl(attn_part_kernel<128>, g1, tpart, 0, st, a);
-    if (e == cudaSuccess) e = launch_pdl(attn_merge_kernel<128>, g2, dim3(128), 0, st, a);
+    if (e == cudaSuccess) e = launch_pdl(attn_merge_kernel<128>, g2, dim3(128 * mg), 0, st, a);
   } else {
     e = launch_pdl(qkv_finish_kernel<64>, gf, dim3(32), 0, st, a);
     if (e == cudaSuccess) e = launch_pdl(attn_part_kernel<64>, g1, tpart, 0, st, a);
-    if (e == cudaSuccess) e = launch_pdl(attn_merge_kernel<64>, g2, dim3(64), 0, st, a);
+    if (e == cudaSuccess) e = launch_pdl(attn_merge_kernel<64>, g2, dim3(64 * mg), 0, st, a);
   }
   return e;
 }
