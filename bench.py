@@ -64,6 +64,8 @@ def parse():
                     help="block sizes k for the verify-time sweep ('' to skip); the budget "
                          "selection needs all of 0..16")
     ap.add_argument("--sweep-blocks", type=int, default=24)
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the 1.5B k-sweep and the ragged 16-request rounds")
     ap.add_argument("--long-kv-len", type=int, default=15128,
                     help="prefix length of the long-context sweep (0 to skip)")
     ap.add_argument("--session", action="store_true",
@@ -384,6 +386,13 @@ def run_ours(args, ws, rank, local):
         long_ctx = None
         if args.long_kv_len > 0 and args.model == "7b":
             long_ctx = measure_long_context(args, lib, D, W, model, cfg, sh, stream, seed)
+        other_cfgs = None
+        if not args.no_configs and args.model == "7b":
+            other_cfgs = {"7b_ragged16": measure_ragged(args, lib, D, model, cfg, sh, stream, seed)}
+            state.close()
+            model.close()
+            torch.cuda.empty_cache()
+            other_cfgs["1.5b_k_sweep"] = measure_1p5b(args, lib, D, sh, stream, seed)
 
     if ws > 1:
         elapsed_ms, committed_all = reduce_ranks(elapsed_ms, committed, "cuda")
@@ -423,6 +432,7 @@ def run_ours(args, ws, rank, local):
     med_us = float(np.median(per_block_us))
     mean_us = elapsed_ms * 1e3 / steps
     step_roof = {"bytes_per_block": int(step_bytes),
+                 "kv_bytes_written_per_block": int((k + 1) * cfg.kv_bytes_per_pos()),
                  "roofline_us": round(step_bytes / (peak * 1e9) * 1e6, 1),
                  "frac_of_mean_block": round(step_bytes / (peak * 1e9) / (mean_us / 1e6), 4),
                  "frac_of_median_block": round(step_bytes / (peak * 1e9) / (med_us / 1e6), 4),
@@ -454,6 +464,7 @@ def run_ours(args, ws, rank, local):
         "budget": budget,
         "prefill": prefill,
         "long_context": long_ctx,
+        "other_configs": other_cfgs,
         "clocks": clk,
         "e2e": e2e,
     }
@@ -461,8 +472,9 @@ def run_ours(args, ws, rank, local):
         line["cpu_baseline"] = cpu_baseline(args, cfg, L0, plans)
     if rank == 0:
         print(json.dumps(line), flush=True)
-    state.close()
-    model.close()
+    if other_cfgs is None:
+        state.close()
+        model.close()
     if ws > 1:
         dist.destroy_process_group()
 
@@ -510,6 +522,101 @@ def measure_long_context(args, lib, D, W, model, cfg, sh, stream, seed, ks=(1, 4
     del kc, vc
     torch.cuda.empty_cache()
     return {"kv_len": L, "blocks_per_k": blocks, "sweep": out}
+
+
+def _timed_blocks(st, cands, ks, sh, stream):
+    """Run one verification call per entry of `cands` (lists of per-request
+    candidate lists) with CUDA events around each; returns (µs per call,
+    committed tokens per call)."""
+    import torch
+    B = len(ks[0])
+    n = torch.zeros(B, dtype=torch.int32, device="cuda")
+    c = torch.zeros(B, dtype=torch.int32, device="cuda")
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in cands]
+    n_all = []
+    torch.cuda.synchronize()
+    for i, (cd, kk) in enumerate(zip(cands, ks)):
+        ev[i][0].record(stream)
+        st.verify(cd, kk, n, c, stream=sh)
+        ev[i][1].record(stream)
+        n_all.append(n.clone())
+    torch.cuda.synchronize()
+    us = [a.elapsed_time(b) * 1e3 for a, b in ev]
+    committed = [int((x + 1).sum().item()) for x in n_all]
+    return us, committed
+
+
+def measure_ragged(args, lib, D, model, cfg, sh, stream, seed, B=16, rounds=128):
+    """The ragged workload: 16 requests with prefixes uniform in [250, 7500] and
+    k uniform in {0..16} per request and round, verified together; uniform
+    candidates (the work of a round does not depend on acceptance)."""
+    import torch
+    rng = np.random.default_rng(seed + 505)
+    lens = [int(x) for x in rng.integers(250, 7501, B)]
+    cap = max(lens) + 17 * rounds + 64
+    kc, vc = D.device_kv(cfg, lens, cap, seed, poison=False)
+    st = lib.State(model, lens, cap, kc, vc, [1] * B)
+    ks = [[int(x) for x in rng.integers(0, 17, B)] for _ in range(rounds)]
+    cands = [torch.from_numpy(rng.integers(0, cfg.vocab, max(sum(kk), 1)).astype(np.int32)).cuda()
+             for kk in ks]
+    _timed_blocks(st, cands[:3], ks[:3], sh, stream)       # warm-up
+    st.rollback(lens, [1] * B, sh)
+    st.read_state(sh)
+    us, committed = _timed_blocks(st, cands, ks, sh, stream)
+    ln, _ = st.read_state(sh)
+    st.check(sh)
+    peak, _ = load_peaks()
+    kv_read = sum((lens[b] + ln[b]) / 2.0 for b in range(B)) * cfg.kv_bytes_per_pos()
+    bts = cfg.weight_bytes() + kv_read
+    mean_us = float(np.mean(us))
+    st.close()
+    del kc, vc
+    torch.cuda.empty_cache()
+    return {"requests": B, "rounds": rounds, "round_us_mean": round(mean_us, 1),
+            "round_us_median": round(float(np.median(us)), 1),
+            "mean_rows_per_round": round(float(np.mean([sum(kk) + B for kk in ks])), 1),
+            "committed_tok_s": round(sum(committed) / (sum(us) / 1e6), 1),
+            "frac": round(bts / (peak * 1e9) / (mean_us / 1e6), 4),
+            "note": "uniform candidates: acceptance (and so committed tok/s) is low; the "
+                    "work of a round does not depend on it"}
+
+
+def measure_1p5b(args, lib, D, sh, stream, seed, L0=814, blocks=24):
+    """The 1.5B-class decoder (814 prefilled positions), verify time versus
+    k in {0, 1, 2, 4, 8}, uniform candidates."""
+    import torch
+    cfg = model_shape("1.5b")
+    w = D.device_weights(cfg, seed)
+    torch.cuda.synchronize()
+    model = lib.Model(cfg, D.weight_pointers(cfg, w))
+    del w
+    torch.cuda.empty_cache()
+    cap = L0 + 9 * (blocks + 2) + 64
+    kc, vc = D.device_kv(cfg, [L0], cap, seed, poison=False)
+    st = lib.State(model, [L0], cap, kc, vc, [1])
+    peak, _ = load_peaks()
+    rng = np.random.default_rng(seed + 606)
+    out = []
+    for k in (0, 1, 2, 4, 8):
+        cands = [torch.from_numpy(rng.integers(0, cfg.vocab, max(k, 1)).astype(np.int32)).cuda()
+                 for _ in range(blocks + 1)]
+        st.rollback([L0], [1], sh)
+        st.read_state(sh)
+        _timed_blocks(st, cands[:1], [[k]], sh, stream)
+        st.rollback([L0], [1], sh)
+        st.read_state(sh)
+        us, _ = _timed_blocks(st, cands[1:], [[k]] * blocks, sh, stream)
+        ln, _ = st.read_state(sh)
+        mean_us = float(np.mean(us))
+        bts = bytes_per_block(cfg, (L0 + ln[0]) / 2.0, k)
+        out.append({"k": k, "verify_us_mean": round(mean_us, 1),
+                    "verify_us_median": round(float(np.median(us)), 1),
+                    "frac": round(bts / (peak * 1e9) / (mean_us / 1e6), 4)})
+    st.check(sh)
+    st.close()
+    model.close()
+    return {"kv_len": L0, "blocks_per_k": blocks, "sweep": out}
 
 
 def measure_prefill(args, lib, W, state, cfg, L0, root0, sh, stream, n_instr=64, reps=5):
