@@ -65,6 +65,9 @@ struct AttnArgs {
   const float* qkv_rinv;  // [qkv_ld] 1 / rms of each token row
   const float2* rope;     // [rows][D / 2] (cos, sin)
   int qkv_split, qkv_ld;
+  // partition items of the split-KV pass, request by request: request b owns
+  // items [part_start[b], part_start[b + 1]) (its own partitions only)
+  int32_t part_start[kMaxBatch + 1];
 };
 
 // ---- finishing the QKV projection from its split-K sums ----------------------

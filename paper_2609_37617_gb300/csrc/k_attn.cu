@@ -36,12 +36,15 @@ template <int D>
 __global__ void __launch_bounds__(256, 1) attn_part_kernel(AttnArgs a) {
   __shared__ __align__(16) bf16 sK[kPart][kPitch];
   __shared__ __align__(16) bf16 sV[kPart][kPitch];
+  // item blockIdx.x -> (request, partition): only each request's own partitions
+  int b = 0;
+  while (b + 1 < a.batch && a.part_start[b + 1] <= (int)blockIdx.x) ++b;
+  const int part = (int)blockIdx.x - a.part_start[b];
   // the keys/values already in the cache do not depend on the predecessor
-  stage_old_kv<D>(a, a.layer, blockIdx.x, blockIdx.y, blockIdx.z, sK, sV, threadIdx.x, blockDim.x);
+  stage_old_kv<D>(a, a.layer, part, blockIdx.y, b, sK, sV, threadIdx.x, blockDim.x);
   ptx::griddep_wait();
   ptx::griddep_launch_dependents();
-  part_item<D, true>(a, a.layer, blockIdx.x, blockIdx.y, blockIdx.z, sK, sV, threadIdx.x,
-                     blockDim.x, 0);
+  part_item<D, true>(a, a.layer, part, blockIdx.y, b, sK, sV, threadIdx.x, blockDim.x, 0);
 }
 
 // The QKV projection finished from its split-K sums (TC_PART): one CTA of
@@ -188,12 +191,15 @@ cudaError_t launch_attention_split(const RowMap& m, const Model& md, KvState& kv
   a.ao = kv.ao;
   a.lo_row = kv.rows_alloc;
   int64_t max_len = 0;
+  a.part_start[0] = 0;
   for (int b = 0; b < kv.batch; ++b) {
     const int64_t e = kv.len_upper[b] + (m.start[b + 1] - m.start[b]);
     max_len = e > max_len ? e : max_len;
+    a.part_start[b + 1] = a.part_start[b] + (int)((e + kPart - 1) / kPart);
   }
   const int parts = (int)((max_len + kPart - 1) / kPart);
-  dim3 g1(parts, c.n_kv_heads, kv.batch);
+  const int items = a.part_start[kv.batch];
+  dim3 g1(items, c.n_kv_heads);
   dim3 g2(m.rows, c.n_q_heads);
   a.qkv_part = kv.qkv_part;
   a.qkv_rinv = kv.qkv_rinv;
@@ -211,7 +217,7 @@ cudaError_t launch_attention_split(const RowMap& m, const Model& md, KvState& kv
   // half the waves.  Which warp takes a row tile does not change its
   // arithmetic.
   int warps = 8;
-  if ((long long)parts * c.n_kv_heads * kv.batch > md.sm_count) {
+  if ((long long)items * c.n_kv_heads > md.sm_count) {
     int qn_max = 0;
     for (int b = 0; b < kv.batch; ++b) {
       const int qn = (m.start[b + 1] - m.start[b]) * (c.n_q_heads / c.n_kv_heads);
