@@ -283,9 +283,10 @@ void as2d_model_free(as2d_model* model);
          cursor moves to j + 1 for the first j in (m, m + W] holding t, else
          to j + 2 for the first j in [m, m + W] holding x, else the target
          decodes alone (k = 0).  While it does, its latest token is looked for
-         before each call in the published positions [s, s + W), s starting
-         at m + 1 and growing by one per token decoded alone; a match at j
-         moves the cursor to j + 1. */
+         before each call in the published positions [s, s + W) upwards, then
+         [max(f, s - W), s) downwards, where f = m + 1 is where it began
+         decoding alone and s starts at f and grows by one per token decoded
+         alone; a match at j moves the cursor to j + 1. */
 #define AS2D_CBUF_BATCH 8
 #define AS2D_CBUF_NORMAL 0   /* candidates follow the cursor              */
 #define AS2D_CBUF_REALIGN 1  /* R1/R2: waiting on the token at m          */
@@ -328,8 +329,16 @@ as2d_status as2d_cbuf_after_call(as2d_cbuf* buf, int32_t k, int32_t n_accepted,
 as2d_status as2d_cbuf_state(as2d_cbuf* buf, int32_t* ready, int32_t* cursor,
                             int32_t* mode);
 
+/* Tokens and batch records the buffer still holds (either may be NULL).
+   Positions stay absolute, but tokens below both the cursor and the
+   alignment position -- which no rule reads again -- are dropped once 4096
+   of them have gathered, with the records of the batches wholly below them
+   (App. C.1: exhausted records are discarded; the others keep their order
+   and provenance), so a long session holds a bounded buffer. */
+as2d_status as2d_cbuf_held(as2d_cbuf* buf, int32_t* tokens, int32_t* records);
+
 /* Copy the source record of the batch that published `position`
-   (AS2D_ERR_INVALID_ARG if the position is not published). */
+   (AS2D_ERR_INVALID_ARG if the position is not published or was dropped). */
 as2d_status as2d_cbuf_source_of(as2d_cbuf* buf, int32_t position,
                                 as2d_source_record* out);
 

@@ -28,11 +28,14 @@ design notes):
       first position j in [m, m + W] holding x (the producer's token after x
       stands in for t, and its continuation after that is verified under
       root t); failing that, the target decodes alone (k = 0).  While it
-      does, its latest token u is the anchor, looked for before each call in
-      the W published positions [s, s + W), s starting at m + 1; a match at
-      j moves the cursor to j + 1, and every token decoded alone retires one
-      more position (s += 1), so the window keeps pace with the target when
-      the producer is behind.
+      does, its latest token u is the anchor, looked for before each call
+      first in the published positions [s, s + W) in increasing order, then
+      in [max(f, s - W), s) from s - 1 down, f = m + 1 being where the
+      target began decoding alone and s starting at f; a match at j moves
+      the cursor to j + 1.  Every token decoded alone advances s by one, so
+      the window keeps pace with the target when the producer is behind, and
+      looking back W positions recovers from deletions in the producer's
+      text (positions below f, or more than W behind s, are retired).
   W is the search bound (default 8).
 Correctness does not depend on any of this: every candidate is verified
 under the current committed prefix, so the committed text is the target's
@@ -68,6 +71,7 @@ class CandidateBuffer:
         self.mode = NORMAL
         self.m = 0             # REALIGN: position of x; ALONE: search start
         self.x = None          # REALIGN: the call's final token; ALONE: the anchor
+        self.f = 0             # ALONE: the first position of the alone search
 
     def publish(self, tokens, record):
         """Append one immutable batch of at most eight tokens."""
@@ -98,7 +102,9 @@ class CandidateBuffer:
         if self.mode == REALIGN and self.m < len(tok) and tok[self.m] == self.x:
             self.cursor, self.mode = self.m + 1, NORMAL
         elif self.mode == ALONE:
-            for j in range(self.m, min(self.m + self.window, len(tok))):
+            ahead = range(self.m, min(self.m + self.window, len(tok)))
+            behind = range(min(self.m, len(tok)) - 1, max(self.f, self.m - self.window) - 1, -1)
+            for j in list(ahead) + list(behind):
                 if tok[j] == self.x:
                     self.cursor, self.mode = j + 1, NORMAL
                     return
@@ -135,6 +141,7 @@ class CandidateBuffer:
                 self.cursor, self.mode = j + 2, NORMAL
                 return
         self.mode, self.m, self.x = ALONE, m + 1, t
+        self.f = self.m
         self.cursor = self.m
 
 

@@ -37,7 +37,7 @@ EXPORTED = ("as2d_model_load", "as2d_kv_init_prefilled", "as2d_verify_block",
             "as2d_model_free", "as2d_last_error", "as2d_kv_profile",
             "as2d_kv_profile_read", "as2d_decode_step_static", "as2d_cbuf_create",
             "as2d_cbuf_publish", "as2d_cbuf_candidates", "as2d_cbuf_after_call",
-            "as2d_cbuf_state", "as2d_cbuf_source_of", "as2d_cbuf_free",
+            "as2d_cbuf_state", "as2d_cbuf_source_of", "as2d_cbuf_free", "as2d_cbuf_held",
             "as2d_verify_from_buffers", "as2d_interval_accounting", "as2d_session_run",
             "as2d_budget_select", "as2d_prefill", "as2d_model_set_sm_budget",
             "as2d_cpu_decoder_create", "as2d_cpu_decoder_step", "as2d_cpu_decoder_logits",
@@ -126,6 +126,8 @@ _lib.as2d_cbuf_candidates.argtypes = [_P, _S, _P, ctypes.POINTER(ctypes.c_int32)
 _lib.as2d_cbuf_after_call.argtypes = [_P, _S, _S, _S]
 _lib.as2d_cbuf_state.argtypes = [_P, _P, _P, _P]
 _lib.as2d_cbuf_source_of.argtypes = [_P, _S, ctypes.POINTER(as2d_source_record)]
+_lib.as2d_cbuf_held.argtypes = [_P, _P, _P]
+_lib.as2d_cbuf_held.restype = _S
 _lib.as2d_cbuf_free.argtypes = [_P]
 _lib.as2d_cbuf_free.restype = None
 _lib.as2d_verify_from_buffers.argtypes = [_P, _P, _S, _P, _P, _P, _P]
@@ -498,6 +500,12 @@ class CandidateBuffer:
         st, ready, cursor, mode = as2d_cbuf_state(self.handle)
         _check(st, "as2d_cbuf_state")
         return ready, cursor, CBUF_MODES[mode]
+
+    def held(self):
+        """(tokens, batch records) the buffer still holds."""
+        t, r = ctypes.c_int32(), ctypes.c_int32()
+        _check(_lib.as2d_cbuf_held(self.handle, ctypes.byref(t), ctypes.byref(r)), "as2d_cbuf_held")
+        return t.value, r.value
 
     def source_of(self, position):
         st, rec = as2d_cbuf_source_of(self.handle, position)

@@ -67,12 +67,19 @@ extern "C" as2d_status as2d_cbuf_state(as2d_cbuf* buf, int32_t* ready, int32_t* 
   return AS2D_OK;
 }
 
+extern "C" as2d_status as2d_cbuf_held(as2d_cbuf* buf, int32_t* tokens, int32_t* records) {
+  clear_error();
+  if (!buf) return report_error(AS2D_ERR_INVALID_ARG, "buf is NULL");
+  buf->b.held(tokens, records);
+  return AS2D_OK;
+}
+
 extern "C" as2d_status as2d_cbuf_source_of(as2d_cbuf* buf, int32_t position,
                                            as2d_source_record* out) {
   clear_error();
   if (!buf || !out) return report_error(AS2D_ERR_INVALID_ARG, "buf and out are required");
   if (!buf->b.source_of(position, out))
-    return report_error(AS2D_ERR_INVALID_ARG, "position is not published");
+    return report_error(AS2D_ERR_INVALID_ARG, "position is not published or was dropped");
   return AS2D_OK;
 }
 

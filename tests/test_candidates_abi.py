@@ -149,3 +149,32 @@ def test_concurrent_publisher(lib):
         L += n + 1
     th.join()
     assert committed == ref[:len(committed)]
+
+
+def test_long_session_holds_a_bounded_buffer(lib):
+    """Long sessions: the library's buffer drops what no rule reads again
+    (positions stay absolute) and still agrees call by call with the
+    oracle's, which keeps everything."""
+    rng = random.Random(99)
+    ref = [rng.randrange(200) for _ in range(30500)]
+    prod = _noisy(ref, rng, 0.05, 0.02, 0.02, 200)
+    _lockstep(lib, ref, prod, lambda i: 64 + 16 * i, 16, 8, 20000)
+    buf = lib.CandidateBuffer()
+    L = 0
+    for i in range(0, 24000, 8):
+        buf.publish(prod[i:i + 8], offset=i)
+    seen_max = 0
+    while L < 20000:
+        c = buf.candidates(16)
+        n, corr = C.verify(ref, L, c)
+        buf.after_call(len(c), n, corr)
+        L += n + 1
+        seen_max = max(seen_max, buf.held()[0])
+    held, recs = buf.held()
+    ready, cursor, _ = buf.state()
+    assert ready == 24000 and cursor > 15000
+    assert held < 24000 - 8000 and recs <= held // 8 + 2
+    with pytest.raises(lib.AS2DError):
+        buf.source_of(0)                      # dropped
+    assert buf.source_of(ready - 1)["offset"] == 24000 - 8
+

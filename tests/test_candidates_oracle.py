@@ -94,6 +94,25 @@ def test_slow_producer_catches_up():
     assert after and all(n == k for k, n, *_ in after) and max(k for k, *_ in after) >= 2
 
 
+def test_alone_search_looks_back_after_a_deletion():
+    """R3: the producer's text lost a token inside the stretch the target
+    decoded alone, so the target's tokens sit one position behind the window
+    start; the look-back finds the anchor and candidates resume."""
+    ref = list(range(100, 200))
+    prod = list(ref)
+    for i in range(1, 12):
+        prod[i] = 900 + i      # junk: the realign search fails, the target decodes alone
+    del prod[5]                # every later position moves back by one
+    calls, comm = C.run_session(ref, prod, lambda i: 10 ** 9, b=4, window=4, target_len=60)
+    assert comm == ref[:len(comm)]
+    modes = [m for *_, m in calls]
+    first_normal_after = next(i for i in range(3, len(calls)) if modes[i] == C.NORMAL)
+    # the anchor 112 sits at position 11 while the window starts at 12
+    assert calls[first_normal_after][3] == 12
+    assert any(n >= 2 for _, n, *_ in calls[first_normal_after:first_normal_after + 3])
+    assert len(calls) < 30
+
+
 def test_batches_are_immutable_and_bounded():
     buf = C.CandidateBuffer()
     with pytest.raises(ValueError):
