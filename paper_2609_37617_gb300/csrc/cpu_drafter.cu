@@ -8,7 +8,8 @@
 // attention over the positions so far, output projection with residual,
 // SwiGLU MLP with residual, final norm, LM head, argmax (lowest index on
 // ties).  Matrix-vector products are split over `threads` OpenMP threads by
-// output rows.
+// output rows, each row's dot product vectorised (a fixed lane order per
+// build).
 #include <cmath>
 #include <new>
 #include <vector>
@@ -48,6 +49,7 @@ void matvec(const float* W, const float* x, float* y, int rows, int cols, int th
   for (int r = 0; r < rows; ++r) {
     const float* w = W + (size_t)r * cols;
     float acc = 0.f;
+#pragma omp simd reduction(+ : acc)
     for (int i = 0; i < cols; ++i) acc += w[i] * x[i];
     y[r] = acc;
   }
