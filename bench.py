@@ -39,9 +39,52 @@ WORKLOAD = "7b"
 
 # dram__bytes_read.sum + dram__bytes_write.sum per launch from one ncu capture
 # of the kernel as it stands (profiles/); None once the kernel has changed.
-# dram bytes per launch from an ncu capture of the current kernel; None when
-# the kernel changed after the capture
 TRAFFIC = {"gate_up": 275262720}  # 271,890,688 read + 3,372,032 written
+
+# Diagnostic legs that reuse the headline state (each rolls it back to L0 first).
+BUDGET_WIN, BUDGET_COMMIT, BUDGET_TRACES = 220, 180, 4
+MAX_K = 16
+
+
+def plan_capacity(L0, k, steps, warmup, sweep_ks, sweep_blocks, committed_plan):
+    """Cache positions the headline state needs, and the length of the greedy
+    trajectory, for every leg that runs on it.  Each leg starts from L0 (a
+    rollback).  Between read-backs the library's host bound of the length
+    grows by k + 1 per call whatever is accepted, and a call is refused once
+    bound + k + 1 exceeds the capacity, so a leg of n calls of width k needs
+    n (k + 1) positions past L0.  Returns (trajectory length, capacity, the
+    positions past L0 of each leg)."""
+    sweep_ks = list(sweep_ks)
+    sweep_need = max(((kk + 1) * sweep_blocks for kk in sweep_ks), default=0)
+    # the trajectory feeds the timed blocks' candidates (up to the planned
+    # committed length + k), the k-sweep's (up to its own advance + k) and
+    # the budget leg's development windows
+    traj_len = max(committed_plan + k + 2, BUDGET_TRACES * BUDGET_WIN + 1,
+                   max(((kk + 1) * sweep_blocks + kk + 1 for kk in sweep_ks), default=0))
+    needs = {
+        "trajectory": traj_len,                    # k = 0 decode steps
+        "warmup": warmup * (k + 1),
+        "timed": steps * (k + 1),                  # also the e2e leg
+        "breakdown": min(8, steps) * (k + 1),
+        "k_sweep": sweep_need,
+        # sessions read every call's outcome back, so the bound stays exact:
+        # the committed tokens plus one call of the widest block
+        "budget": BUDGET_COMMIT + 2 * (MAX_K + 1),
+        "prefill": 0,                              # rewrites positions below L0
+    }
+    return traj_len, L0 + max(needs.values()) + 64, needs
+
+
+def guarded(errors, name, fn, *a, **kw):
+    """Run one diagnostic leg; a failure is recorded under `name` in `errors`
+    (and reported as None) instead of ending the run."""
+    import traceback
+    try:
+        return fn(*a, **kw)
+    except Exception as exc:  # noqa: BLE001 -- every leg failure is reported, not raised
+        errors[name] = f"{type(exc).__name__}: {exc}"
+        traceback.print_exc(file=sys.stderr)
+        return None
 
 
 def parse():
@@ -54,10 +97,9 @@ def parse():
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--profile-class", default="auto",
-                    help="kernel class timed live for the roofline; auto = the whole "
-                         "persistent pass when it is enabled (AS2D_PERSISTENT=1, "
-                         "k + 1 <= 32 rows), else gate_up")
+    ap.add_argument("--profile-class", default="gate_up",
+                    help="kernel class timed live for the roofline (the dominant one, "
+                         "gate_up, by default)")
     ap.add_argument("--model", default="7b", help="model shape (7b; smaller ones for quick checks)")
     ap.add_argument("--kv-len", type=int, default=1564)
     ap.add_argument("--sweep", default=",".join(str(i) for i in range(17)),
@@ -208,8 +250,9 @@ def run_ours(args, ws, rank, local):
         torch.cuda.empty_cache()
         plans = draw_plans(args, steps, cfg.vocab)
         committed_plan = int((plans[:, 0] + 1).sum())
-        traj_len = committed_plan + k + 2
-        cap = L0 + (k + 1) * max(steps, warm) + traj_len + 64
+        sweep_ks = [int(x) for x in args.sweep.split(",") if x != ""] if args.sweep else []
+        traj_len, cap, _ = plan_capacity(L0, k, steps, warm, sweep_ks, args.sweep_blocks,
+                                         committed_plan)
         kc, vc = D.device_kv(cfg, [L0], cap, seed, poison=False)
         root0 = int(W.root_tokens(cfg, 1, seed)[0])
         state = lib.State(model, [L0], cap, kc, vc, [root0])
@@ -299,48 +342,59 @@ def run_ours(args, ws, rank, local):
         n_np = n_all.cpu().numpy()
         committed = int((n_np + 1).sum())
         plan_match = float(np.mean(n_np == plans[:, 0]))
+        # everything below is diagnostic: a leg that fails is reported in the
+        # line's "errors" instead of ending the run
+        errors = {}
         # pass 2: the same blocks again with event pairs around every launch of
         # the dominant kernel class, for its live average duration
         prof_cls = args.profile_class
-        if prof_cls == "auto":
-            prof_cls = "pass" if (k + 1) <= 32 and os.environ.get("AS2D_PERSISTENT", "0") == "1" else "gate_up"
-        # run twice and keep the faster: a transient stall of the shared host
-        # would otherwise set the kernel's figure
-        prof = []
-        for _ in range(2):
-            pn, pms, _ = timed_pass(prof_cls)
-            prof.append((pms / pn if pn else float("inf"), pn, pms, t0.elapsed_time(t1)))
-        _, prof_n, prof_ms, pass2_ms = min(prof)
-        state.check(sh)
-        # pass 3 (diagnostic): an event pair around every block for the
-        # distribution of block times
-        timed_pass(None, per_block=True)
-        per_block_us = np.array([a.elapsed_time(b) * 1e3 for a, b in ev])
-        state.check(sh)
 
-        # per-class device time per block (diagnostic, after the timed region)
-        breakdown = {}
-        for cls_name in ("qkv", "attention", "o", "gate_up", "down", "lm_head", "other", "pass"):
-            state.rollback([L0], [root0], sh)
-            state.read_state(sh)
-            state.profile(cls_name)
-            state.profile_read()
-            nb_blocks = min(8, steps)
-            for i in range(nb_blocks):
-                block(i, i)
-            n_cls, ms_cls, _ = state.profile_read()
-            if n_cls:
-                breakdown[cls_name] = round(ms_cls / nb_blocks * 1e3, 1)
-        state.profile(None)
-        state.check(sh)
+        def pass2():
+            # run twice and keep the faster: a transient stall of the shared
+            # host would otherwise set the kernel's figure
+            prof = []
+            for _ in range(2):
+                pn, pms, _ = timed_pass(prof_cls)
+                prof.append((pms / pn if pn else float("inf"), pn, pms, t0.elapsed_time(t1)))
+            state.check(sh)
+            return min(prof)[1:]
 
-        # verify time and committed tokens/s versus k (same acceptance law,
-        # capped at k), and the per-position cost reduction R(K) of Eq. 2
-        sweep = []
-        if args.sweep:
-            ks = [int(x) for x in args.sweep.split(",") if x != ""]
+        prof_n, prof_ms, pass2_ms = guarded(errors, "kernel_timing", pass2) or (0, 0.0, 0.0)
+
+        def pass3():
+            # an event pair around every block for the distribution of block times
+            timed_pass(None, per_block=True)
+            state.check(sh)
+            return np.array([a.elapsed_time(b) * 1e3 for a, b in ev])
+
+        per_block_us = guarded(errors, "per_block", pass3)
+
+        def class_breakdown():
+            # per-class device time per block (after the timed region)
+            breakdown = {}
+            for cls_name in ("qkv", "attention", "o", "gate_up", "down", "lm_head", "other"):
+                state.rollback([L0], [root0], sh)
+                state.read_state(sh)
+                state.profile(cls_name)
+                state.profile_read()
+                nb_blocks = min(8, steps)
+                for i in range(nb_blocks):
+                    block(i, i)
+                n_cls, ms_cls, _ = state.profile_read()
+                if n_cls:
+                    breakdown[cls_name] = round(ms_cls / nb_blocks * 1e3, 1)
+            state.profile(None)
+            state.check(sh)
+            return breakdown
+
+        breakdown = guarded(errors, "class_us_per_block", class_breakdown)
+
+        def k_sweep():
+            # verify time and committed tokens/s versus k (same acceptance law,
+            # capped at k), and the per-position cost reduction R(K) of Eq. 2
+            sweep = []
             nbk = args.sweep_blocks
-            for kk in ks:
+            for kk in sweep_ks:
                 pl = draw_plans(args, nbk, cfg.vocab, k=kk, seed_offset=1000 + kk) if kk > 0 else None
                 pl_d = torch.from_numpy(pl.astype(np.int32)).cuda() if kk > 0 else None
                 cand_k = torch.zeros(max(kk, 1), dtype=torch.int32, device="cuda")
@@ -357,7 +411,8 @@ def run_ours(args, ws, rank, local):
                         rc = synth._load_cuda().synth_cuda_build_candidates(
                             cand_k.data_ptr(), traj.data_ptr(), traj_len + 1, len_dev, L0,
                             pl_d[i].data_ptr(), kk, cfg.vocab, sh)
-                        assert rc == 0
+                        if rc != 0:
+                            raise RuntimeError(f"synth_cuda_build_candidates returned {rc}")
                     out = lib.make_verify_out(nk.data_ptr() + 4 * i, ck.data_ptr() + 4 * i)
                     lib._check(lib.as2d_verify_block(state.handle, cand_k.data_ptr() if kk else 0,
                                                      [kk], out, sh), "as2d_verify_block")
@@ -374,25 +429,33 @@ def run_ours(args, ws, rank, local):
             if v1:
                 for e in sweep:
                     e["R_pct"] = round(100.0 * (1.0 - e["verify_us_mean"] / (e["K"] * v1)), 1)
+            return sweep
+
+        sweep = (guarded(errors, "k_sweep", k_sweep) or []) if sweep_ks else []
 
         budget = None
-        if len(sweep) == 17 and [e["k"] for e in sweep] == list(range(17)):
-            budget = select_budget(args, lib, state, traj, sweep, cfg, L0, root0, sh)
+        if len(sweep) == MAX_K + 1 and [e["k"] for e in sweep] == list(range(MAX_K + 1)):
+            budget = guarded(errors, "budget", select_budget, args, lib, state, traj, sweep, cfg,
+                             L0, root0, sh)
 
         e2e = None
         if not args.no_e2e:
-            e2e = run_e2e(args, lib, W, state, traj, plans, cfg, L0, root0, sh, stream)
-        prefill = measure_prefill(args, lib, W, state, cfg, L0, root0, sh, stream)
+            e2e = guarded(errors, "e2e", run_e2e, args, lib, W, state, traj, plans, cfg, L0,
+                          root0, sh, stream)
+        prefill = guarded(errors, "prefill", measure_prefill, args, lib, W, state, cfg, L0,
+                          root0, sh, stream)
         long_ctx = None
         if args.long_kv_len > 0 and args.model == "7b":
-            long_ctx = measure_long_context(args, lib, D, W, model, cfg, sh, stream, seed)
+            long_ctx = guarded(errors, "long_context", measure_long_context, args, lib, D, W,
+                               model, cfg, sh, stream, seed)
         other_cfgs = None
         if not args.no_configs and args.model == "7b":
-            other_cfgs = {"7b_ragged16": measure_ragged(args, lib, D, model, cfg, sh, stream, seed)}
-            state.close()
-            model.close()
+            other_cfgs = {"7b_ragged16": guarded(errors, "7b_ragged16", measure_ragged, args, lib,
+                                                 D, model, cfg, sh, stream, seed)}
+            guarded(errors, "close_7b", lambda: (state.close(), model.close()))
             torch.cuda.empty_cache()
-            other_cfgs["1.5b_k_sweep"] = measure_1p5b(args, lib, D, sh, stream, seed)
+            other_cfgs["1.5b_k_sweep"] = guarded(errors, "1.5b_k_sweep", measure_1p5b, args, lib,
+                                                 D, sh, stream, seed)
 
     if ws > 1:
         elapsed_ms, committed_all = reduce_ranks(elapsed_ms, committed, "cuda")
@@ -407,7 +470,6 @@ def run_ours(args, ws, rank, local):
     cls = prof_cls
     mean_len = L0 + committed / 2.0
     per_unit = {
-        "pass": bytes_per_block(cfg, mean_len, k),
         "gate_up": 2 * F * H * 2 + rows * (H * 4 + 2 * H * 2 + F * 2),
         "down": H * F * 2 + rows * (F * 2 + 2 * H * 4),
         "qkv": (cfg.n_q + 2 * cfg.n_kv) * cfg.head_dim * H * 2 + rows * (H * 4 + 2 * H * 2),
@@ -429,15 +491,21 @@ def run_ours(args, ws, rank, local):
                                 "event pairs; the faster of two such passes); value comes "
                                 "from the first pass, without them"}
     step_bytes = bytes_per_block(cfg, L0 + committed / 2.0, k)  # mean length over the blocks
-    med_us = float(np.median(per_block_us))
     mean_us = elapsed_ms * 1e3 / steps
+    med_us = float(np.median(per_block_us)) if per_block_us is not None else None
     step_roof = {"bytes_per_block": int(step_bytes),
                  "kv_bytes_written_per_block": int((k + 1) * cfg.kv_bytes_per_pos()),
                  "roofline_us": round(step_bytes / (peak * 1e9) * 1e6, 1),
                  "frac_of_mean_block": round(step_bytes / (peak * 1e9) / (mean_us / 1e6), 4),
-                 "frac_of_median_block": round(step_bytes / (peak * 1e9) / (med_us / 1e6), 4),
+                 "frac_of_median_block": (round(step_bytes / (peak * 1e9) / (med_us / 1e6), 4)
+                                          if med_us else None),
                  "note": "mean over the headline pass (no event between blocks); median from "
                          "a diagnostic pass with an event pair around every block"}
+    verify_us = None
+    if per_block_us is not None:
+        verify_us = {"mean": round(mean_us, 1), "median": round(med_us, 1),
+                     "p10": round(float(np.percentile(per_block_us, 10)), 1),
+                     "p90": round(float(np.percentile(per_block_us, 90)), 1)}
 
     line = {
         "metric": METRIC, "value": round(value, 2), "unit": UNIT, "n_gpus": ws,
@@ -446,12 +514,11 @@ def run_ours(args, ws, rank, local):
         "dtype": "bf16", "data": "synthetic (seeded random-init weights and KV; greedy-derived candidates)",
         "config": {"workload": f"{args.model} verify, k={k}, L0={L0}, {steps} consecutive blocks, "
                                "geometric acceptance (mean 3, capped at k)",
-                   "k": k, "kv_len": L0, "blocks": steps, "batch": 1,
+                   "k": k, "kv_len": L0, "blocks": steps, "batch": 1, "capacity": cap,
                    "l2": f"inputs larger than L2 ({cfg.weight_bytes() / 1e9:.2f} GB of weights "
                          "streamed per step)",
                    "parallelism": f"replicas x{ws}" if ws > 1 else "single GPU"},
-        "verify_us": {"median": round(med_us, 1), "p10": round(float(np.percentile(per_block_us, 10)), 1),
-                      "p90": round(float(np.percentile(per_block_us, 90)), 1)},
+        "verify_us": verify_us,
         "mean_committed_per_block": round(committed / steps, 3),
         "plan_match": plan_match,
         "step_roofline": step_roof,
@@ -467,14 +534,15 @@ def run_ours(args, ws, rank, local):
         "other_configs": other_cfgs,
         "clocks": clk,
         "e2e": e2e,
+        "errors": errors or None,
     }
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(args, cfg, L0, plans)
+        line["cpu_baseline"] = guarded(errors, "cpu_baseline", cpu_baseline, args, cfg, L0, plans)
+        line["errors"] = errors or None
     if rank == 0:
         print(json.dumps(line), flush=True)
     if other_cfgs is None:
-        state.close()
-        model.close()
+        guarded(errors, "close", lambda: (state.close(), model.close()))
     if ws > 1:
         dist.destroy_process_group()
 
@@ -726,8 +794,9 @@ def run_e2e(args, lib, W, state, traj, plans, cfg, L0, root0, sh, stream):
 
 
 def cpu_baseline(args, cfg, L0, plans):
-    """The CPU oracle (as it stands) on one verification block of the same
-    workload: one k-block forward at L0 on the host cores."""
+    """The CPU oracle (as it stands) on the same workload, on the host cores:
+    one k-block forward at L0 with every core (OpenMP over output rows), and
+    one decode row (one of the block's k + 1 rows) on a single thread."""
     import oracle
     from synth import workloads as W
     k = args.k
@@ -737,16 +806,32 @@ def cpu_baseline(args, cfg, L0, plans):
     cache = om.cache(ks, vs)
     root = int(W.root_tokens(cfg, 1, args.seed)[0])
     cand = plans[0, 2:2 + k]
-    t0 = time.perf_counter()
-    om.verify_block(cache, L0, root, cand, want_logits=False)
-    dt = time.perf_counter() - t0
     mean_committed = float((plans[:, 0] + 1).mean())
-    cores = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    default_threads = oracle.set_threads(0)
+    try:
+        cores = oracle.set_threads(default_threads)
+        t0 = time.perf_counter()
+        om.verify_block(cache, L0, root, cand, want_logits=False)
+        dt = time.perf_counter() - t0
+        # one row single-threaded, at the block's last position (the rows of a
+        # block cost the same up to the few extra keys)
+        oracle.set_threads(1)
+        t0 = time.perf_counter()
+        om.decode_step(cache, L0, root)
+        dt1 = time.perf_counter() - t0
+    finally:
+        oracle.set_threads(default_threads)
+    v1 = mean_committed / (dt1 * (k + 1))
     return {"value": round(mean_committed / dt, 4), "unit": UNIT, "cores": cores,
             "kind": "oracle",
             "sample": f"one k={k} verification block of the {cfg.name} decoder at L={L0} "
-                      f"({dt:.2f} s, fp64, OpenMP); value = mean committed tokens per block "
-                      "of the timed plan / that block time"}
+                      f"({dt:.2f} s, fp64, OpenMP over output rows on {cores} threads); value = "
+                      "mean committed tokens per block of the timed plan / that block time",
+            "single_thread": {"value": round(v1, 4), "unit": UNIT, "cores": 1,
+                              "sample": f"one decode row at L={L0} on one thread ({dt1:.2f} s); "
+                                        f"value = mean committed tokens per block / ({k + 1} x "
+                                        "that row time)"},
+            "host_cores": os.cpu_count()}
 
 
 def run_reference(args, ws, rank):
@@ -778,7 +863,7 @@ def run_reference(args, ws, rank):
     rows_per_s = steps / dt
     mean_committed = float((plans[:, 0] + 1).mean())
     value = rows_per_s * mean_committed / (k + 1)
-    cores = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    cores = oracle.set_threads(0)
     line = {"impl": "reference", "metric": METRIC, "value": round(value, 4), "unit": UNIT,
             "n_gpus": ws, "steps": steps, "warmup": warm,
             "ms_per_step": round(dt / steps * 1e3, 3), "higher_is_better": True,

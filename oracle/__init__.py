@@ -62,8 +62,16 @@ def load(precision="f64"):
                                             _P, _P, _P, _P, _P, _P, _P]
         lib.oracle_verify_block.restype = _I32
         lib.oracle_real_bytes.restype = _I32
+        lib.oracle_set_threads.argtypes = [_I32]
+        lib.oracle_set_threads.restype = _I32
         _LIBS[precision] = lib
     return _LIBS[precision]
+
+
+def set_threads(n, precision="f64"):
+    """Threads of the oracle's OpenMP loops (n <= 0: the default); returns
+    the count in effect.  The thread count changes no result."""
+    return int(load(precision).oracle_set_threads(int(n)))
 
 
 def _ptr(a):

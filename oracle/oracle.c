@@ -13,6 +13,7 @@
 #include "oracle.h"
 
 #include <math.h>
+#include <omp.h>
 #include <stdlib.h>
 #include <string.h>
 
@@ -22,6 +23,11 @@
 typedef ORACLE_REAL real;
 
 int32_t oracle_real_bytes(void) { return (int32_t)sizeof(real); }
+
+int32_t oracle_set_threads(int32_t n) {
+  if (n > 0) omp_set_num_threads(n);
+  return (int32_t)omp_get_max_threads();
+}
 
 /* ---- bf16 conversions ------------------------------------------------- */
 

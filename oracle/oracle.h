@@ -103,6 +103,11 @@ int32_t oracle_verify_block(const oracle_config* cfg, const oracle_weights* w,
                             int32_t* greedy, double* logits, double* margin,
                             int64_t* new_len, int32_t* new_root);
 
+/* Threads of the OpenMP loops (over independent output rows and heads; the
+   count changes no sum's order).  n <= 0 leaves the runtime's default.
+   Returns the count the next parallel loop will use. */
+int32_t oracle_set_threads(int32_t n);
+
 /* sizeof(ORACLE_REAL) this build computes in (8 or 4). */
 int32_t oracle_real_bytes(void);
 
