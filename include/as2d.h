@@ -49,6 +49,15 @@ typedef int32_t as2d_status;
 #define AS2D_ERR_DEVICE (-5)        /* a kernel reported an error or timeout */
 #define AS2D_ERR_NO_MEMORY (-6)     /* a host allocation failed              */
 
+/* Device-side error bits (as2d_kv_check's message names them; the static
+   decode step returns them through its error_bits output). */
+#define AS2D_DEVERR_BAD_TOKEN 1  /* a root or candidate id outside [0, vocab)  */
+#define AS2D_DEVERR_ROLLBACK 2   /* a rollback beyond the committed length     */
+#define AS2D_DEVERR_TIMEOUT 4    /* a kernel's bounded wait gave up            */
+#define AS2D_DEVERR_CAPACITY 8   /* a device-side length left no room for the
+                                    call's rows (length < 0 or length + rows >
+                                    capacity): that request was skipped       */
+
 /* Largest number of candidates per request in one call (the budget b of
    App. A.2; physical width K = k + 1 <= 17). */
 #define AS2D_MAX_K 16
@@ -210,22 +219,31 @@ as2d_status as2d_kv_check(as2d_kv* kv, void* stream);
    k_cache, v_cache: device bf16 [n_layers][1][n_kv][capacity][head_dim] as
    for as2d_kv_init_prefilled.  len, root: device int32 [1], the request's
    state, updated in place (len += 1, root = correction) as by
-   as2d_decode_step.  correction_token: device int32 [1].  logits: device
-   float [vocab] or NULL.
+   as2d_decode_step; *len must lie in [0, capacity - 1] when the step runs.
+   correction_token: device int32 [1].  logits: device float [vocab] or NULL.
+   error_bits: device int32 [1] or NULL; receives the step's AS2D_DEVERR_*
+   bits (0 when it ran cleanly).
    Limits (AS2D_ERR_CAPACITY / AS2D_ERR_UNSUPPORTED on the host, before any
    work): capacity <= 4096, hidden <= 4096, ffn <= 20480, n_q * head_dim <=
    4096, n_kv <= 8, n_q / n_kv <= 16, vocab <= 262144, at most 192 SMs.
+   The length lives on the device, so the host cannot check it: the kernels
+   do.  A step whose *len is outside [0, capacity - 1], or whose root is
+   outside [0, vocab), writes nothing to the cache, leaves len and root as
+   they were, sets *correction_token to -1 and reports AS2D_DEVERR_CAPACITY
+   (or AS2D_DEVERR_BAD_TOKEN) in error_bits.
    The first call on a device (and the first after a model of another shape)
    looks up the array's device address and builds descriptors of it; make
-   that first call before any stream capture.  All calls share the one
-   array and each call starts by clearing the parts that must start at zero,
-   so calls that overlap on the GPU (other streams, other host threads) race
-   and give wrong results: issue them one after another.  Device-side
-   errors of this entry point are not reported through as2d_kv_check. */
+   that first call before any stream capture.  Calls from several host
+   threads are enqueued one at a time, but all calls share the one array and
+   each starts by clearing the parts that must start at zero, so calls that
+   overlap on the GPU (other streams) race and give wrong results: issue
+   them one after another on one stream, or synchronise between them.
+   Device-side errors of this entry point are reported only through
+   error_bits, not through as2d_kv_check. */
 as2d_status as2d_decode_step_static(as2d_model* model, void* k_cache, void* v_cache,
                                     int32_t capacity, int32_t* len, int32_t* root,
                                     int32_t* correction_token, float* logits,
-                                    void* stream);
+                                    int32_t* error_bits, void* stream);
 
 /* Measurement support (not part of the verification step).  Kernel classes
    of one verification pass, in launch order per layer: */
@@ -236,10 +254,7 @@ as2d_status as2d_decode_step_static(as2d_model* model, void* k_cache, void* v_ca
 #define AS2D_KERNEL_DOWN 4       /* down projection + residual          */
 #define AS2D_KERNEL_LM_HEAD 5    /* final norm + LM head + argmax       */
 #define AS2D_KERNEL_OTHER 6      /* embedding gather, accept scan, ...  */
-#define AS2D_KERNEL_PASS 7       /* the whole pass as one persistent kernel
-                                    (opt-in: AS2D_PERSISTENT=1; calls of
-                                    at most 32 rows)                     */
-#define AS2D_KERNEL_CLASSES 8
+#define AS2D_KERNEL_CLASSES 7
 
 /* Record a CUDA event pair on the call's stream around the launches of
    kernel class `kernel_class` (one pair per layer, or per call for the LM

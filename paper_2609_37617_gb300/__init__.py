@@ -26,6 +26,10 @@ AS2D_ERR_CUDA = -3
 AS2D_ERR_UNSUPPORTED = -4
 AS2D_ERR_DEVICE = -5
 AS2D_ERR_NO_MEMORY = -6
+AS2D_DEVERR_BAD_TOKEN = 1
+AS2D_DEVERR_ROLLBACK = 2
+AS2D_DEVERR_TIMEOUT = 4
+AS2D_DEVERR_CAPACITY = 8
 AS2D_CBUF_BATCH = 8
 CBUF_MODES = {0: "normal", 1: "realign", 2: "alone"}
 AS2D_MAX_K = 16
@@ -43,7 +47,7 @@ EXPORTED = ("as2d_model_load", "as2d_kv_init_prefilled", "as2d_verify_block",
             "as2d_cpu_decoder_create", "as2d_cpu_decoder_step", "as2d_cpu_decoder_logits",
             "as2d_cpu_decoder_reset", "as2d_cpu_decoder_free")
 KERNEL_CLASSES = {"qkv": 0, "attention": 1, "o": 2, "gate_up": 3, "down": 4,
-                  "lm_head": 5, "other": 6, "pass": 7}
+                  "lm_head": 5, "other": 6}
 
 
 class as2d_config(ctypes.Structure):
@@ -118,7 +122,7 @@ _lib.as2d_kv_profile_read.argtypes = [_P, ctypes.POINTER(ctypes.c_int32),
                                       ctypes.POINTER(ctypes.c_double),
                                       ctypes.POINTER(ctypes.c_int64)]
 _lib.as2d_kv_profile_read.restype = _S
-_lib.as2d_decode_step_static.argtypes = [_P, _P, _P, ctypes.c_int32, _P, _P, _P, _P, _P]
+_lib.as2d_decode_step_static.argtypes = [_P, _P, _P, ctypes.c_int32, _P, _P, _P, _P, _P, _P]
 _lib.as2d_decode_step_static.restype = _S
 _lib.as2d_cbuf_create.argtypes = [_S, ctypes.POINTER(ctypes.c_void_p)]
 _lib.as2d_cbuf_publish.argtypes = [_P, _P, _S, ctypes.POINTER(as2d_source_record)]
@@ -270,12 +274,13 @@ def as2d_kv_profile_read(kv):
 
 
 def as2d_decode_step_static(model, k_cache_ptr, v_cache_ptr, capacity, len_ptr, root_ptr,
-                            correction_ptr, logits_ptr=0, stream=0):
+                            correction_ptr, logits_ptr=0, error_bits_ptr=0, stream=0):
     """Single-request decode step whose working memory is the library's fixed
     array (no allocation); see include/as2d.h."""
     return _lib.as2d_decode_step_static(_P(model), _P(int(k_cache_ptr)), _P(int(v_cache_ptr)),
                                         int(capacity), _P(int(len_ptr)), _P(int(root_ptr)),
                                         _P(int(correction_ptr)), _P(int(logits_ptr) or None),
+                                        _P(int(error_bits_ptr) or None),
                                         _P(int(stream) or None))
 
 

@@ -3,6 +3,7 @@
 // verification pass (Section 3.2; App. C.2).
 #include <cstdlib>
 #include <cstring>
+#include <mutex>
 #include <string>
 
 #include "as2d_internal.h"
@@ -340,13 +341,6 @@ extern "C" as2d_status as2d_kv_init_prefilled(as2d_model* mh, int32_t batch,
   }
   cudaError_t e;
   const size_t bytes = s.work_bytes;
-  e = mk_prepare(m, s);
-  if (e != cudaSuccess) {
-    cudaFree(s.mk_mem);
-    cudaFree(s.work);
-    delete kh;
-    return fail(AS2D_ERR_CUDA, std::string("preparing the persistent pass: ") + cudaGetErrorString(e));
-  }
   e = cudaMemset(s.work, 0, bytes);
   if (e == cudaSuccess)
     e = cudaMalloc(&s.rope_full, (size_t)capacity * (m.cfg.head_dim / 2) * sizeof(float2));
@@ -356,7 +350,6 @@ extern "C" as2d_status as2d_kv_init_prefilled(as2d_model* mh, int32_t batch,
   if (e == cudaSuccess) e = cudaDeviceSynchronize();
   if (e != cudaSuccess) {
     cudaFree(s.rope_full);
-    cudaFree(s.mk_mem);
     cudaFree(s.work);
     delete kh;
     return fail(AS2D_ERR_CUDA, std::string("initialising the state: ") + cudaGetErrorString(e));
@@ -368,7 +361,6 @@ extern "C" as2d_status as2d_kv_init_prefilled(as2d_model* mh, int32_t batch,
 extern "C" void as2d_kv_free(as2d_kv* kh) {
   if (!kh) return;
   for (cudaEvent_t e : kh->s.prof_events) cudaEventDestroy(e);
-  cudaFree(kh->s.mk_mem);
   cudaFree(kh->s.work);
   cudaFree(kh->s.rope_full);
   cudaFree(kh->s.cb_dev);
@@ -475,7 +467,6 @@ cudaError_t tc_project(int epi, const Model& m, KvState& s, const RowMap& rm, co
     const CUtensorMap& x = xmaps[nb_index(nb)];
     cudaError_t e;
     switch (epi) {
-      case TC_QKV: e = tc_gemm_qkv(nb, x, p, st); break;
       case TC_PART: e = tc_gemm_part(nb, x, p, st); break;
       case TC_RESID: e = tc_gemm_resid(nb, x, p, st); break;
       case TC_SWIGLU: e = tc_gemm_swiglu(nb, x, p, st); break;
@@ -518,14 +509,7 @@ as2d_status run_block(KvState& s, const int32_t* cand, const int32_t* k,
   // One pass of the verification step (Section 3.2; App. C.2): embedding
   // gather, n_layers x {QKV (split-K sums), RoPE + KV append + attention, O + residual,
   // gate/up + SwiGLU, down + residual}, LM head + argmax, accept scan, as a
-  // sequence of kernels chained by programmatic dependent launch.  With
-  // AS2D_PERSISTENT=1 in the environment, calls of at most 32 rows run it as
-  // one persistent kernel instead (same arithmetic, same results).
-  if (!force && !root_override && mk_usable(s, rm.rows)) {
-    LAUNCH(AS2D_KERNEL_PASS, launch_mk(rm, m, s, cand, *out, st));
-    for (int b = 0; b < s.batch; ++b) s.len_upper[b] += (k ? k[b] : 0) + 1;
-    return AS2D_OK;
-  }
+  // sequence of kernels chained by programmatic dependent launch.
   LAUNCH(AS2D_KERNEL_OTHER, launch_embed(rm, m, s, cand, st, root_override));
   TcParams tp{};
   tp.h = s.h;
@@ -706,6 +690,7 @@ extern "C" as2d_status as2d_kv_check(as2d_kv* kh, void* stream) {
     if (err & kErrBadToken) msg += " candidate or root token outside [0, vocab);";
     if (err & kErrRollback) msg += " rollback beyond the committed length;";
     if (err & kErrTimeout) msg += " a kernel wait timed out;";
+    if (err & kErrCapacity) msg += " a device-side length left no room for the call's rows;";
     return fail(AS2D_ERR_DEVICE, msg);
   }
   return AS2D_OK;
@@ -802,6 +787,9 @@ KvState make_static_state() {
   return s;
 }
 KvState g_static_kv = make_static_state();
+// Guards g_static_dev and g_static_kv: calls from several host threads are
+// enqueued one at a time (their work on the GPU still shares one array).
+std::mutex g_static_mu;
 
 }  // namespace
 
@@ -811,7 +799,7 @@ static __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBy
 extern "C" as2d_status as2d_decode_step_static(as2d_model* mh, void* k_cache, void* v_cache,
                                                int32_t capacity, int32_t* len, int32_t* root,
                                                int32_t* correction_token, float* logits,
-                                               void* stream) {
+                                               int32_t* error_bits, void* stream) {
   g_err.clear();
   if (!mh || !k_cache || !v_cache || !len || !root || !correction_token)
     return fail(AS2D_ERR_INVALID_ARG, "model, caches, len, root and correction_token are required");
@@ -830,6 +818,7 @@ extern "C" as2d_status as2d_decode_step_static(as2d_model* mh, void* k_cache, vo
   CUDA_TRY(cudaGetDevice(&dev));
   if (dev < 0 || dev >= kStaticMaxDevices)
     return fail(AS2D_ERR_UNSUPPORTED, "device ordinal above 63");
+  std::lock_guard<std::mutex> lock(g_static_mu);
   StaticDevice& sd = g_static_dev[dev];
   if (!sd.ready || sd.hidden != c.hidden || sd.q_dim != m.q_dim || sd.ffn != c.ffn) {
     // Set-up, once per device (and again only if a model of another shape is
@@ -885,10 +874,13 @@ extern "C" as2d_status as2d_decode_step_static(as2d_model* mh, void* k_cache, vo
   s.tm_u[0] = sd.tm_u;
   s.prof_class = -1;
   // the array keeps the previous call's contents: clear the error words, the
-  // argmax slots and the stream-K arrival counters, which must start at zero
+  // argmax slots and the stream-K arrival counters (as many as the largest
+  // projection has tiles, as for an allocated state), which must start at zero
+  const int wide = c.vocab > 2 * c.ffn ? c.vocab : 2 * c.ffn;
+  s.n_counters = (wide + 127) / 128 + 64;
   CUDA_TRY(cudaMemsetAsync(b + kOffErr, 0, 256, st));
   CUDA_TRY(cudaMemsetAsync(b + kOffBest, 0, kStaticRows * 8, st));
-  CUDA_TRY(cudaMemsetAsync(b + kOffCnt, 0, (size_t)(c.vocab / 128 + 64) * 4, st));
+  CUDA_TRY(cudaMemsetAsync(b + kOffCnt, 0, (size_t)s.n_counters * 4, st));
 
   RowMap rm;
   rm.batch = 1;
@@ -932,7 +924,12 @@ extern "C" as2d_status as2d_decode_step_static(as2d_model* mh, void* k_cache, vo
   }
   LAUNCH(AS2D_KERNEL_LM_HEAD, tc_project(TC_LOGITS, m, s, rm, m.lm_head, s.tm_xn, c.vocab, H, tp, st));
   LAUNCH(AS2D_KERNEL_OTHER, launch_accept(rm, m, s, nullptr, out, st));
+  // the call's device error bits, for the caller (a copy, not an allocation)
+  if (error_bits)
+    CUDA_TRY(cudaMemcpyAsync(error_bits, b + kOffErr, sizeof(int32_t), cudaMemcpyDeviceToDevice, st));
   return AS2D_OK;
 }
 
+static_assert(kStaticMaxVocab / 128 + 64 >= (2 * kStaticMaxFfn) / 128 + 64,
+              "the counter region covers the largest projection's tiles");
 static_assert(kStaticScratchBytes == 12930048, "as2d.h states the fixed working-memory size");

@@ -36,14 +36,26 @@ __host__ __device__ inline int row_request(const RowMap& m, int r) {
   return b;
 }
 
-// Device error bits (ORed into KvState::d_err).
+// Device error bits (ORed into KvState::d_err); the values of include/as2d.h's
+// AS2D_DEVERR_* bits.
 enum : int32_t {
-  kErrBadToken = 1,
-  kErrRollback = 2,
-  kErrTimeout = 4,
+  kErrBadToken = AS2D_DEVERR_BAD_TOKEN,
+  kErrRollback = AS2D_DEVERR_ROLLBACK,
+  kErrTimeout = AS2D_DEVERR_TIMEOUT,
+  kErrCapacity = AS2D_DEVERR_CAPACITY,
 };
 
-enum TcEpi { TC_QKV = 0, TC_RESID = 1, TC_SWIGLU = 2, TC_LOGITS = 3, TC_PART = 4 };
+// Whether a request of device-side length `len` has room for `rows` more
+// cache entries.  A request that does not is skipped by every kernel that
+// indexes the cache or the rotary table with its length (no key/value append,
+// no attention, zero attention output); the embedding kernel flags it
+// (kErrCapacity and the request's bad flag), and the accept scan then reports
+// n_accepted = correction = -1 and leaves its length and root unchanged.
+__host__ __device__ inline bool rows_fit(int len, int rows, int cap) {
+  return len >= 0 && len <= cap - rows;
+}
+
+enum TcEpi { TC_RESID = 1, TC_SWIGLU = 2, TC_LOGITS = 3, TC_PART = 4 };
 
 struct TcParams {
   const bf16* w;         // packed weight blocks (k_pack.cu), unit u at u * 8192
@@ -176,12 +188,6 @@ struct KvState {
   int attn_qmax = 0;         // (kMaxK + 1) * group, rounded up to 16
   // TMA descriptors of the activation operands, per token-row padding
   CUtensorMap tm_xn[kNbCount], tm_ao[kNbCount], tm_u[kNbCount];
-  // persistent single-launch pass (k_mk.cu)
-  bool mk_ok = false;
-  void* mk_mem = nullptr;          // phase table, then per-phase arrival counters
-  unsigned int* mk_bar = nullptr;
-  int mk_n_phases = 0;
-  unsigned int mk_gen = 0;         // calls so far
   // measurement support
   int prof_class = -1;
   std::vector<cudaEvent_t> prof_events;  // pairs
@@ -224,17 +230,9 @@ int attn_partitions(int capacity);
 cudaError_t launch_attention_split(const RowMap& m, const Model& md, KvState& kv, int layer,
                                    cudaStream_t st);
 
-// Persistent single-launch pass for calls of at most 32 rows (k_mk.cu).
-cudaError_t mk_prepare(const Model& m, KvState& kv);
-bool mk_usable(const KvState& kv, int rows);
-cudaError_t launch_mk(const RowMap& rm, const Model& m, KvState& kv, const int32_t* cand,
-                      const as2d_verify_out& out, cudaStream_t st);
-
 // Tensor-core GEMM launchers (k_tc_*.cu), one per fused epilogue.
 int qkv_split_for(const Model& m);
 cudaError_t tc_gemm_part(int nb, const CUtensorMap& x, const TcParams& p, cudaStream_t st);
-cudaError_t tc_gemm_qkv(int nb, const CUtensorMap& x, const TcParams& p,
-                        cudaStream_t st);
 cudaError_t tc_gemm_resid(int nb, const CUtensorMap& x, const TcParams& p,
                           cudaStream_t st);
 cudaError_t tc_gemm_swiglu(int nb, const CUtensorMap& x, const TcParams& p,

@@ -32,8 +32,7 @@
 //     K evenly over a fixed number of CTAs per tile and stores each CTA's
 //     unscaled sums: the attention's first kernel adds them, applies RoPE and
 //     appends the keys and values, so no CTA of this kernel waits for
-//     another's part at its end.  (TC_QKV, the same epilogue done here by the
-//     last CTA of a tile, serves the persistent whole-pass kernel.)
+//     another's part at its end.
 // Every mbarrier wait is bounded in time; on expiry the kernel records an
 // error bit, drains its own outstanding copies and MMAs, frees TMEM and exits.
 #pragma once
@@ -106,13 +105,11 @@ __device__ __forceinline__ int tc_owner(long long u, const TcParams& p) {
 }
 
 // Operands of one 16-row epilogue chunk that come from memory (the residual
-// and the norm gain for RESID, the rotary table for QKV), fetched by
-// tc_epilogue_load before they are needed so that their loads overlap other
-// loads of the caller.
+// and the norm gain for RESID), fetched by tc_epilogue_load before they are
+// needed so that their loads overlap other loads of the caller.
 struct TcEpiIn {
   float hv[16];
   float gn;
-  float2 cs[16];
 };
 
 template <int NB, int EPI>
@@ -125,15 +122,6 @@ __device__ __forceinline__ void tc_epilogue_load(const TcParams& p, TcEpiIn& in,
 #pragma unroll
     for (int j = 0; j < CH; ++j)
       if (m0 + j < p.rows) in.hv[j] = p.h[(size_t)(p.row0 + m0 + j) * p.N + col];
-  } else if (EPI == TC_QKV) {
-    const int d = p.d, half = d >> 1;
-    const int head = col / d, e = col - head * d;
-    const int i = e < half ? e : e - half;
-    if (head < p.nq + p.nkv) {
-#pragma unroll
-      for (int j = 0; j < CH; ++j)
-        if (m0 + j < p.rows) in.cs[j] = p.rope[(size_t)(p.row0 + m0 + j) * half + i];
-    }
   }
 }
 
@@ -192,42 +180,6 @@ __device__ __forceinline__ void tc_epilogue_apply(const TcParams& p, const TcEpi
       const size_t at = (size_t)(p.row0 + m) * F + (size_t)tile * 64 + i;
       p.u[at] = uh;
       p.u[at + (size_t)p.lo_row * F] = __float2bfloat16_rn(uv - __bfloat162float(uh));
-    }
-  } else if (EPI == TC_QKV) {
-    // thread et owns tile row n = et (one element of one head) for the chunk's
-    // 16 token rows
-    const int d = p.d, half = d >> 1, q_dim = p.nq * d;
-    const int n = et, col = tile * 128 + n, head = col / d, e = col - head * d;
-    const int partner = e < half ? n + half : n - half;
-    const bool rotate = head < p.nq + p.nkv;
-    const float2* cs = in.cs;
-    int pos[CH];
-#pragma unroll
-    for (int j = 0; j < CH; ++j)
-      if (m0 + j < p.rows) pos[j] = s_pos[m0 + j];
-#pragma unroll
-    for (int j = 0; j < CH; ++j) {
-      const int m = m0 + j;
-      if (m >= p.rows) break;
-      const int gm = p.row0 + m;
-      const float x = sC[n * SP + j];
-      if (rotate) {
-        const float xp = sC[partner * SP + j];
-        const float y = (e < half) ? x * cs[j].x - xp * cs[j].y : x * cs[j].x + xp * cs[j].y;
-        if (head < p.nq) {
-          p.q[(size_t)gm * q_dim + col] = y;
-        } else {
-          const int b = s_req[m];
-          const size_t off =
-              ((((size_t)p.layer * p.batch + b) * p.nkv + (head - p.nq)) * p.cap + pos[j]) * d + e;
-          p.kc[off] = __float2bfloat16_rn(y);
-        }
-      } else {
-        const int b = s_req[m];
-        const size_t off =
-            ((((size_t)p.layer * p.batch + b) * p.nkv + (head - p.nq - p.nkv)) * p.cap + pos[j]) * d + e;
-        p.vc[off] = __float2bfloat16_rn(x);
-      }
     }
   } else {  // TC_LOGITS
     if (p.logits) {
@@ -293,11 +245,6 @@ __device__ __forceinline__ void tc_row_prologue(const TcParams& p, float* s_rinv
     // round trip for up to 32 tiles' sums (hidden <= 4096)
     for (int m = et; m < p.rows; m += 128) {
       const int gm = p.row0 + m;
-      int len_b = 0, b = 0;
-      if (EPI == TC_QKV) {
-        b = row_request(p.rm, gm);
-        len_b = p.len[b];
-      }
       if (EPI != TC_RESID) {
         // 1 / rms of the token row from the producer's per-tile sums (in order)
         const float* src = p.ss + gm;
@@ -313,10 +260,6 @@ __device__ __forceinline__ void tc_row_prologue(const TcParams& p, float* s_rinv
         s_rinv[m] = rsqrtf(tot / (float)p.hidden + p.eps);
         // TC_PART leaves the scaling to the kernel that finishes its sums
         if (EPI == TC_PART && blockIdx.x == 0) p.part_rinv[gm] = s_rinv[m];
-      }
-      if (EPI == TC_QKV) {
-        s_req[m] = b;
-        s_pos[m] = len_b + (gm - p.rm.start[b]);
       }
     }
     if (EPI != TC_RESID) ptx::named_bar_sync(1, 128);

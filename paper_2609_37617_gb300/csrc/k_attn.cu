@@ -40,10 +40,12 @@ __global__ void __launch_bounds__(256, 1) attn_part_kernel(AttnArgs a) {
   int b = 0;
   while (b + 1 < a.batch && a.part_start[b + 1] <= (int)blockIdx.x) ++b;
   const int part = (int)blockIdx.x - a.part_start[b];
+  const bool fits = rows_fit(a.len[b], a.rm.start[b + 1] - a.rm.start[b], a.cap);
   // the keys/values already in the cache do not depend on the predecessor
-  stage_old_kv<D>(a, a.layer, part, blockIdx.y, b, sK, sV, threadIdx.x, blockDim.x);
+  if (fits) stage_old_kv<D>(a, a.layer, part, blockIdx.y, b, sK, sV, threadIdx.x, blockDim.x);
   ptx::griddep_wait();
   ptx::griddep_launch_dependents();
+  if (!fits) return;  // flagged by the embedding kernel; nothing of the cache is read
   part_item<D, true>(a, a.layer, part, blockIdx.y, b, sK, sV, threadIdx.x, blockDim.x, 0);
 }
 
@@ -59,6 +61,7 @@ __global__ void __launch_bounds__(D / 2) qkv_finish_kernel(AttnArgs a) {
   constexpr int H2 = D / 2;
   const int gm = blockIdx.x, head = blockIdx.y, e = threadIdx.x;
   const int b = row_request(a.rm, gm), pos = a.len[b] + (gm - a.rm.start[b]);
+  if (!rows_fit(a.len[b], a.rm.start[b + 1] - a.rm.start[b], a.cap)) return;  // no append
   const float2 y = (head < a.nq + a.nkv) ? qk_rotated<D>(a, head, e, gm)
                                          : make_float2(qkv_value(a, head * D + e, gm),
                                                        qkv_value(a, head * D + e + H2, gm));
@@ -102,6 +105,14 @@ __global__ void __launch_bounds__(kMergeGroups * D) attn_merge_kernel(AttnArgs a
   const int b = row_request(a.rm, r);
   const int i = r - a.rm.start[b];
   const int g = j / G, qr = i * G + (j - g * G);
+  if (!rows_fit(a.len[b], a.rm.start[b + 1] - a.rm.start[b], a.cap)) {
+    // a skipped request: zero output, no partition is read
+    for (int e = tid; e < D; e += nthr) {
+      a.ao[(size_t)r * a.nq * D + (size_t)j * D + e] = __float2bfloat16_rn(0.f);
+      a.ao[(size_t)(a.lo_row + r) * a.nq * D + (size_t)j * D + e] = __float2bfloat16_rn(0.f);
+    }
+    return;
+  }
   const int pos = a.len[b] + i;
   const int nparts = pos / kPart + 1;
   const size_t base = (size_t)(b * a.nkv + g) * a.parts_max * a.qmax + qr;

@@ -36,17 +36,24 @@ __global__ void rope_table_kernel(float2* __restrict__ out, int d, double theta)
 __global__ void __launch_bounds__(128) embed_kernel(
     RowMap m, const int32_t* __restrict__ cand, const int32_t* __restrict__ root,
     const int32_t* __restrict__ root_override, const bf16* __restrict__ E, int H, int V, float* __restrict__ h, int32_t* err, int32_t* bad,
-    const int32_t* __restrict__ len, float2* __restrict__ rope, const float2* __restrict__ rope_full,
-    int d, double theta, const float* __restrict__ g0, bf16* __restrict__ xn,
-    float* __restrict__ ss, int ss_ld) {
+    const int32_t* __restrict__ len, int cap, float2* __restrict__ rope,
+    const float2* __restrict__ rope_full, int d, double theta, const float* __restrict__ g0,
+    bf16* __restrict__ xn, float* __restrict__ ss, int ss_ld) {
   ptx::griddep_wait();
   ptx::griddep_launch_dependents();
   __shared__ float part[4];
   const int r = blockIdx.x;
   const int b = row_request(m, r);
   const int i = r - m.start[b];
+  // a request whose length leaves no room for its rows is flagged and skipped
+  // downstream (rows_fit); its rows take position 0's rotary entries
+  const bool fits = rows_fit(len[b], m.start[b + 1] - m.start[b], cap);
+  if (!fits && threadIdx.x == 0) {
+    atomicOr(err, kErrCapacity);
+    bad[b] = 1;
+  }
   if ((int)threadIdx.x < d / 2) {
-    const int e = threadIdx.x, pos = len[b] + i;
+    const int e = threadIdx.x, pos = fits ? len[b] + i : 0;
     rope[(size_t)r * (d / 2) + e] =
         rope_full ? rope_full[(size_t)pos * (d / 2) + e] : rope_angle(pos, e, d, theta);
   }
@@ -107,7 +114,7 @@ cudaError_t launch_embed(const RowMap& m, const Model& md, KvState& kv,
   return launch_pdl(embed_kernel, dim3(m.rows), dim3(128), 0, st, m, cand,
                     (const int32_t*)kv.d_root, root_override, (const bf16*)md.embed, md.cfg.hidden,
                     md.cfg.vocab, kv.h, kv.d_err, kv.d_err + 1, (const int32_t*)kv.d_len,
-                    kv.rope, (const float2*)kv.rope_full, md.cfg.head_dim,
+                    kv.capacity, kv.rope, (const float2*)kv.rope_full, md.cfg.head_dim,
                     (double)md.cfg.rope_theta, md.attn_norm[0], kv.xn, kv.ss, kv.rows_alloc);
 }
 
