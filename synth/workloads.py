@@ -99,10 +99,14 @@ class WeightSpec:
 
 def weight_specs(cfg, gains="unit", sigma=0.02, gain_sigma=0.1):
     """All tensors of a model.  gains="unit" gives RMSNorm gains of exactly 1.0
-    (the workloads' reading); gains="random" draws 1 + N(0, gain_sigma)."""
-    gs, gb = (0.0, 1.0) if gains == "unit" else (gain_sigma, 1.0)
+    (the workloads' reading); gains="random" draws 1 + N(0, gain_sigma);
+    gains="sharp" keeps the layer gains at 1.0 and sets the final norm's gain
+    to 8.0, which scales every logit by 8: the same arithmetic with greedy
+    decisions separated by wider margins (the exactness tests use it)."""
+    gs, gb = (0.0, 1.0) if gains in ("unit", "sharp") else (gain_sigma, 1.0)
+    fb = 8.0 if gains == "sharp" else gb
     specs = [WeightSpec("embed", (cfg.vocab, cfg.hidden), S_EMBED, sigma, 0.0),
-             WeightSpec("final_norm", (cfg.hidden,), S_FINAL_NORM, gs, gb),
+             WeightSpec("final_norm", (cfg.hidden,), S_FINAL_NORM, gs, fb),
              WeightSpec("lm_head", (cfg.vocab, cfg.hidden), S_LM_HEAD, sigma, 0.0)]
     for l in range(cfg.n_layers):
         for kind in LAYER_KINDS:

@@ -66,7 +66,22 @@ def run_gpu_block(st, cfg, cand_lists, want_logits=True):
             logits.cpu().numpy() if want_logits else None)
 
 
-def compare_block(oracle_res, gpu_logits, gpu_greedy, gpu_n, gpu_corr, k):
+class ExactTally:
+    """How many bit-exact comparisons actually ran: greedy tokens compared on
+    rows whose oracle margin exceeds MARGIN_SURE, and (n_accepted,
+    correction) pairs compared on blocks whose deciding rows all do.  A test
+    module asserts at the end that its exact half was not skipped."""
+
+    def __init__(self):
+        self.rows = 0
+        self.blocks = 0
+
+    def assert_ran(self, rows=1, blocks=1):
+        assert self.rows >= rows and self.blocks >= blocks, (
+            f"bit-exact checks ran on {self.rows} rows and {self.blocks} blocks only")
+
+
+def compare_block(oracle_res, gpu_logits, gpu_greedy, gpu_n, gpu_corr, k, tally=None):
     """Parity rule: logits within LOGIT_TOL everywhere; greedy tokens equal
     where the oracle's margin exceeds MARGIN_SURE; n_accepted and the
     correction equal whenever every margin they depend on exceeds it."""
@@ -75,9 +90,26 @@ def compare_block(oracle_res, gpu_logits, gpu_greedy, gpu_n, gpu_corr, k):
     sure = oracle_res["margin"] > MARGIN_SURE
     assert np.array_equal(oracle_res["greedy"][sure], gpu_greedy[sure])
     n = oracle_res["n_accepted"]
-    if np.all(sure[: n + 1]):
+    exact = bool(np.all(sure[: n + 1]))
+    if exact:
         assert gpu_n == n and gpu_corr == oracle_res["correction"]
+    if tally is not None:
+        tally.rows += int(sure.sum())
+        tally.blocks += int(exact)
     return d
+
+
+def sharp_root(oracle_model, cache_fn, length, n, start=0, limit=400):
+    """The first root token, searching upward from `start`, whose n-token
+    oracle greedy continuation from `length` has every top-1 minus top-2
+    margin above MARGIN_SURE (cache_fn() gives a fresh oracle cache).  Returns
+    (root, continuation, margins).  A search on the oracle only."""
+    import oracle
+    for root in range(start, start + limit):
+        cont, m = oracle.greedy_continuation(oracle_model, cache_fn(), length, root, n)
+        if np.all(np.asarray(m) > MARGIN_SURE):
+            return root, cont, m
+    raise AssertionError("no root with well-separated greedy decisions found")
 
 
 def oracle_block(pair, cache, length, root, cand):
@@ -85,9 +117,12 @@ def oracle_block(pair, cache, length, root, cand):
     return pair.oracle.verify_block(cache, length, root, list(cand))
 
 
-def check_parity(ores, gpu, row0, k, where=""):
-    """Compare one request's oracle result with its rows of a GPU call
-    (gpu = (n, corr, greedy, logits) arrays; request at row offset row0)."""
+def check_parity(ores, gpu, row0, k, where="", tally=None, b=0):
+    """Compare request b's oracle result with its rows of a GPU call (gpu =
+    (n, corr, greedy, logits) arrays; the request's rows start at row0):
+    logits within LOGIT_TOL, greedy tokens where the margin is sure, and
+    n_accepted / correction when every row they depend on is sure.  Returns
+    (max |dlogit|, whether the commit was compared, oracle n, oracle corr)."""
     n, corr, greedy, logits = gpu
     d = np.max(np.abs(ores["logits"] - logits[row0:row0 + k + 1]))
     assert d <= LOGIT_TOL, f"{where}: max |dlogit| = {d}"
@@ -95,4 +130,10 @@ def check_parity(ores, gpu, row0, k, where=""):
     g = greedy[row0:row0 + k + 1]
     assert np.array_equal(ores["greedy"][sure], g[sure]), where
     m = ores["n_accepted"]
-    return d, bool(np.all(sure[: m + 1])), m, ores["correction"]
+    exact = bool(np.all(sure[: m + 1]))
+    if exact:
+        assert n[b] == m and corr[b] == ores["correction"], where
+    if tally is not None:
+        tally.rows += int(sure.sum())
+        tally.blocks += int(exact)
+    return d, exact, m, ores["correction"]

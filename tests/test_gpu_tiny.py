@@ -7,11 +7,13 @@ import pytest
 
 import oracle
 from synth import workloads as W
-from tests.helpers import Pair, bf16_bits, compare_block, run_gpu_block
+from tests.helpers import (ExactTally, Pair, bf16_bits, compare_block, run_gpu_block,
+                           sharp_root)
 
 pytestmark = pytest.mark.gpu
 
 L0, CAP = 200, 256
+TALLY = ExactTally()
 
 
 @pytest.fixture(scope="module")
@@ -20,6 +22,25 @@ def pair():
     if not torch.cuda.is_available():
         pytest.skip("no GPU")
     return Pair(W.TINY, seed=0)
+
+
+@pytest.fixture(scope="module")
+def pair_sharp():
+    """The tiny shape with the final norm's gain at 8 (logits x 8), so that
+    greedy decisions are separated by more than the 0.1 margin."""
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no GPU")
+    return Pair(W.TINY, seed=0, gains="sharp")
+
+
+@pytest.fixture(scope="module")
+def sharp_continuation(pair_sharp):
+    """Searched on the oracle: the first root whose 9-token greedy
+    continuation from 200 positions has every margin above 0.1."""
+    p = pair_sharp
+    root, cont, margins = sharp_root(p.oracle, lambda: p.oracle_cache(L0, CAP), L0, 9)
+    return root, cont, margins
 
 
 @pytest.fixture(scope="module")
@@ -63,7 +84,7 @@ def test_tiny_block_parity(which, request):
     ores = p.oracle.verify_block(oc, L0, root, cand)
     st = p.state([L0], CAP, [root])
     n, corr, greedy, logits = run_gpu_block(st, cfg, [cand])
-    compare_block(ores, logits[:5], greedy[:5], n[0], corr[0], 4)
+    compare_block(ores, logits[:5], greedy[:5], n[0], corr[0], 4, TALLY)
     ln, rt = st.read_state()
     assert ln == [L0 + n[0] + 1] and rt == [corr[0]]
     # the KV entries kept for the committed rows match the oracle's
@@ -78,16 +99,40 @@ def test_tiny_block_parity(which, request):
     st.close()
 
 
-def test_full_acceptance_and_bonus(pair):
-    cfg = pair.cfg
-    root = int(W.root_tokens(cfg, 1, 0)[0])
-    oc = pair.oracle_cache(L0, CAP)
-    cont, margins = oracle.greedy_continuation(pair.oracle, oc, L0, root, 8)
-    st = pair.state([L0], CAP, [root])
-    n, corr, greedy, _ = run_gpu_block(st, cfg, [cont], want_logits=False)
-    if np.all(margins > 0.1):
-        assert n[0] == 8 and corr[0] == oracle.greedy_continuation(
-            pair.oracle, oc, L0, root, 9)[0][8]
+def test_full_acceptance_and_bonus(pair_sharp, sharp_continuation):
+    """Invariant I1 (Prop. 1): candidates equal to the target's own greedy
+    continuation are all accepted and the correction is the bonus token.
+    Every margin of the continuation exceeds 0.1, so this is asserted
+    unconditionally."""
+    cfg = pair_sharp.cfg
+    root, cont, margins = sharp_continuation
+    assert np.all(np.asarray(margins) > 0.1)
+    st = pair_sharp.state([L0], CAP, [root])
+    n, corr, greedy, _ = run_gpu_block(st, cfg, [cont[:8]], want_logits=False)
+    assert n[0] == 8 and corr[0] == cont[8]
+    assert np.array_equal(greedy, np.asarray(cont[:9]))
+    TALLY.rows += 9
+    TALLY.blocks += 1
+    ln, rt = st.read_state()
+    assert ln == [L0 + 9] and rt == [cont[8]]
+    st.close()
+
+
+def test_sharp_workload_block(pair_sharp, sharp_continuation):
+    """The workload's block shape (k = 4, place 2 replaced) on the sharp
+    model: the rejection at place 2 and its correction are compared bit for
+    bit, since every row they depend on has a margin above 0.1."""
+    cfg = pair_sharp.cfg
+    root, cont, _ = sharp_continuation
+    cand = W.replace_at(cont[:4], 2, np.random.default_rng(0), cfg.vocab)
+    oc = pair_sharp.oracle_cache(L0, CAP)
+    ores = pair_sharp.oracle.verify_block(oc, L0, root, cand)
+    assert ores["n_accepted"] == 2 and ores["correction"] == cont[2]
+    st = pair_sharp.state([L0], CAP, [root])
+    n, corr, greedy, logits = run_gpu_block(st, cfg, [cand])
+    blocks = TALLY.blocks
+    compare_block(ores, logits[:5], greedy[:5], n[0], corr[0], 4, TALLY)
+    assert TALLY.blocks == blocks + 1
     st.close()
 
 
@@ -269,3 +314,9 @@ def test_max_batch_max_k_and_capacity_edge(pair):
     st.check()
     single.close()
     st.close()
+
+
+def test_zz_exact_checks_ran():
+    """The module's bit-exact half ran: greedy rows and at least one full
+    (n_accepted, correction) comparison (the sharp-model blocks above)."""
+    TALLY.assert_ran(rows=9, blocks=2)

@@ -49,3 +49,30 @@ def test_offset_gains(built):
     g = synth.normal_bf16(4096, 0, 3, sigma=0.1, base=1.0)
     f = (g.astype(np.uint32) << 16).view(np.float32)
     assert abs(f.mean() - 1.0) < 0.01
+
+
+def test_sharp_gains_scale_only_the_final_norm():
+    """gains="sharp": layer gains stay 1.0, the final norm's gain is 8.0
+    (exact in bf16), every other tensor is the unit-gain model's."""
+    from synth import workloads as W
+    unit = W.host_weights(W.TINY, 0)
+    sharp = W.host_weights(W.TINY, 0, gains="sharp")
+    assert np.all(sharp["final_norm"] == 0x4100)          # 8.0 in bf16
+    for name in unit:
+        if name != "final_norm":
+            assert np.array_equal(unit[name], sharp[name]), name
+
+
+def test_sharp_root_search_finds_separated_decisions():
+    """The exactness tests' root search, on the oracle only: on the sharp tiny
+    model it finds a root whose 9-token greedy continuation from 200
+    positions has every margin above 0.1 (the unit-gain model's margins are
+    mostly below it)."""
+    import oracle
+    from synth import workloads as W
+    from tests.helpers import MARGIN_SURE, sharp_root
+    cfg = W.TINY
+    om = oracle.Model(cfg, W.host_weights(cfg, 0, gains="sharp"))
+    ks, vs = W.host_kv_request(cfg, 0, 200, 256, 0)
+    root, cont, m = sharp_root(om, lambda: om.cache(ks, vs), 200, 9)
+    assert len(cont) == 9 and np.all(np.asarray(m) > MARGIN_SURE)
