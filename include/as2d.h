@@ -214,7 +214,7 @@ as2d_status as2d_kv_check(as2d_kv* kv, void* stream);
    a real-time loop that cannot accept the latency or the possible failure of
    an allocation.  The model must have been loaded (as2d_model_load allocates,
    once, at set-up).  Every other byte a call needs lives in one array of
-   12,930,048 bytes compiled into the library; each GPU that loads the library
+   9,735,424 bytes compiled into the library; each GPU that loads the library
    holds it until the process exits.
    k_cache, v_cache: device bf16 [n_layers][1][n_kv][capacity][head_dim] as
    for as2d_kv_init_prefilled.  len, root: device int32 [1], the request's

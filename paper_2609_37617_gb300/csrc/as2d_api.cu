@@ -75,6 +75,23 @@ bool encode_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t oute
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+}  // namespace
+
+bool as2d::encode_cache_map(CUtensorMap* map, const void* cache, int head_dim, int capacity,
+                            int64_t heads) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[3] = {(cuuint64_t)head_dim, (cuuint64_t)capacity, (cuuint64_t)heads};
+  cuuint64_t strides[2] = {(cuuint64_t)head_dim * 2, (cuuint64_t)capacity * head_dim * 2};
+  cuuint32_t box[3] = {64, 128, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(cache), dims, strides,
+            box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+namespace {
+
 as2d_status check_config(const as2d_config* c) {
   if (!c) return fail(AS2D_ERR_INVALID_ARG, "config is NULL");
   if (c->n_layers <= 0 || c->hidden <= 0 || c->n_q_heads <= 0 ||
@@ -247,7 +264,6 @@ as2d_status alloc_work(KvState& s, const Model& m, int batch, int capacity,
   const size_t max_tiles = ((size_t)(m.cfg.vocab > 2 * F ? m.cfg.vocab : 2 * F) + 127) / 128 + 64;
   size_t bytes = 4096 + 3 * align_up((size_t)(batch + 1) * 4, 256);
   bytes += align_up(R * H * 4, 256) + align_up(2 * R * H * 2, 256) +
-           align_up(R * m.q_dim * 4, 256) +
            align_up(2 * R * m.q_dim * 2, 256) + align_up(2 * R * F * 2, 256) + align_up(R * 8, 256) +
            align_up(R * (m.cfg.head_dim / 2) * 8, 256) + align_up(R * (H / 128) * 4, 256) +
            align_up((size_t)m.sm_count * 2 * s.nb_max * 128 * 4, 256) + align_up(max_tiles * 4, 256);
@@ -255,10 +271,13 @@ as2d_status alloc_work(KvState& s, const Model& m, int batch, int capacity,
   const size_t qkv_tiles = (size_t)(m.qkv_rows + 127) / 128;
   bytes += align_up(qkv_tiles * s.qkv_split * R * 128 * 4, 256) + align_up(R * 4, 256);
   const int group = m.cfg.n_q_heads / m.cfg.n_kv_heads;
-  s.attn_parts = attn_partitions(capacity);
-  s.attn_qmax = (rows_per_request * group + 15) / 16 * 16;
-  const size_t attn_rows = (size_t)batch * m.cfg.n_kv_heads * s.attn_parts * s.attn_qmax;
-  bytes += align_up(attn_rows * m.cfg.head_dim * 4, 256) + align_up(attn_rows * 8, 256);
+  s.attn_qt = attn_q_tiles(rows_per_request, group);
+  s.attn_chunks = attn_chunks(capacity);
+  const size_t attn_items = (size_t)batch * m.cfg.n_kv_heads * s.attn_qt;
+  const size_t attn_rows = attn_items * s.attn_chunks * 64;
+  bytes += align_up(attn_items * attn_qimg_bytes(m.cfg.head_dim), 256) +
+           align_up(attn_rows * m.cfg.head_dim * 4, 256) + align_up(attn_rows * 8, 256) +
+           align_up(attn_items * 8 * 4, 256);
   cudaError_t e = cudaMalloc(&s.work, bytes);
   if (e != cudaSuccess) {
     s.work = nullptr;
@@ -271,7 +290,6 @@ as2d_status alloc_work(KvState& s, const Model& m, int batch, int capacity,
   s.d_err = cv.take<int32_t>(batch + 1);
   s.h = cv.take<float>(R * H);
   s.xn = cv.take<bf16>(2 * R * H);
-  s.q = cv.take<float>(R * m.q_dim);
   s.ao = cv.take<bf16>(2 * R * m.q_dim);
   s.u = cv.take<bf16>(2 * R * F);
   s.best = cv.take<unsigned long long>(R);
@@ -283,9 +301,15 @@ as2d_status alloc_work(KvState& s, const Model& m, int batch, int capacity,
   s.n_counters = (int)max_tiles;
   s.qkv_part = cv.take<float>(qkv_tiles * s.qkv_split * R * 128);
   s.qkv_rinv = cv.take<float>(R);
+  s.qimg = cv.take<uint8_t>(attn_items * attn_qimg_bytes(m.cfg.head_dim));
   s.attn_o = cv.take<float>(attn_rows * m.cfg.head_dim);
   s.attn_ml = cv.take<float2>(attn_rows);
-  bool ok = true;
+  s.attn_cnt = cv.take<int>(attn_items * 8);
+  s.n_attn_cnt = (int)attn_items * 8;
+  bool ok = encode_cache_map(&s.tm_kc, s.k_cache, m.cfg.head_dim, capacity,
+                             (int64_t)m.cfg.n_layers * batch * m.cfg.n_kv_heads) &&
+            encode_cache_map(&s.tm_vc, s.v_cache, m.cfg.head_dim, capacity,
+                             (int64_t)m.cfg.n_layers * batch * m.cfg.n_kv_heads);
   for (int i = 0; i < kNbCount && ok; ++i) {
     const int nb = 16 << i;
     if (nb > s.nb_max) break;
@@ -296,7 +320,7 @@ as2d_status alloc_work(KvState& s, const Model& m, int batch, int capacity,
   if (!ok) {
     cudaFree(s.work);
     s.work = nullptr;
-    return fail(AS2D_ERR_CUDA, "cuTensorMapEncodeTiled failed for an activation buffer");
+    return fail(AS2D_ERR_CUDA, "cuTensorMapEncodeTiled failed for an activation buffer or a cache");
   }
   return AS2D_OK;
 }
@@ -514,16 +538,6 @@ as2d_status run_block(KvState& s, const int32_t* cand, const int32_t* k,
   TcParams tp{};
   tp.h = s.h;
   tp.u = s.u;
-  tp.q = s.q;
-  tp.kc = s.k_cache;
-  tp.vc = s.v_cache;
-  tp.rope = s.rope;
-  tp.len = s.d_len;
-  tp.batch = s.batch;
-  tp.cap = s.capacity;
-  tp.nq = c.n_q_heads;
-  tp.nkv = c.n_kv_heads;
-  tp.d = c.head_dim;
   tp.logits = out->logits;
   tp.best = s.best;
   tp.xn = s.xn;
@@ -535,11 +549,12 @@ as2d_status run_block(KvState& s, const int32_t* cand, const int32_t* k,
   tp.hidden = c.hidden;
   const int H = c.hidden, F = c.ffn;
   for (int l = 0; l < c.n_layers; ++l) {
-    tp.layer = l;
     LAUNCH(AS2D_KERNEL_QKV, tc_project(TC_PART, m, s, rm, m.w_qkv[l], s.tm_xn, m.qkv_rows, H, tp, st));
     LAUNCH(AS2D_KERNEL_ATTENTION, launch_attention_split(rm, m, s, l, st));
     tp.g_next = m.mlp_norm[l];
+    tp.small_ring = 1;
     LAUNCH(AS2D_KERNEL_O, tc_project(TC_RESID, m, s, rm, m.w_o[l], s.tm_ao, H, m.q_dim, tp, st));
+    tp.small_ring = 0;
     LAUNCH(AS2D_KERNEL_GATE_UP, tc_project(TC_SWIGLU, m, s, rm, m.w_gu[l], s.tm_xn, 2 * F, H, tp, st));
     tp.g_next = (l + 1 < c.n_layers) ? m.attn_norm[l + 1] : m.final_norm;
     LAUNCH(AS2D_KERNEL_DOWN, tc_project(TC_RESID, m, s, rm, m.w_down[l], s.tm_u, H, F, tp, st));
@@ -686,6 +701,8 @@ extern "C" as2d_status as2d_kv_check(as2d_kv* kh, void* stream) {
     // a kernel that gave up may have left split-tile arrival counts behind
     if (kh->s.counters && kh->s.n_counters > 0)
       CUDA_TRY(cudaMemset(kh->s.counters, 0, (size_t)kh->s.n_counters * 4));
+    if (kh->s.attn_cnt && kh->s.n_attn_cnt > 0)
+      CUDA_TRY(cudaMemset(kh->s.attn_cnt, 0, (size_t)kh->s.n_attn_cnt * 4));
     std::string msg = "device error:";
     if (err & kErrBadToken) msg += " candidate or root token outside [0, vocab);";
     if (err & kErrRollback) msg += " rollback beyond the committed length;";
@@ -747,14 +764,15 @@ constexpr int kStaticMaxCapacity = 4096;
 constexpr int kStaticMaxVocab = 262144;
 constexpr int kStaticMaxSms = 192;
 constexpr int kStaticRows = 16;          // one token row, padded to a TMA box
-constexpr int kStaticParts = kStaticMaxCapacity / 64;
+constexpr int kStaticChunks = kStaticMaxCapacity / 1024;  // attention chunks
 
 constexpr size_t sa(size_t x) { return (x + 255) / 256 * 256; }
 constexpr size_t kOffErr = 0;                                                     // err, bad, n
 constexpr size_t kOffH = kOffErr + 256;
 constexpr size_t kOffXn = kOffH + sa((size_t)kStaticRows * kStaticMaxHidden * 4);
+// one query tile per kv head (a single row of at most 16 query heads per group)
 constexpr size_t kOffQ = kOffXn + sa((size_t)2 * kStaticRows * kStaticMaxHidden * 2);
-constexpr size_t kOffAo = kOffQ + sa((size_t)kStaticRows * kStaticMaxQDim * 4);
+constexpr size_t kOffAo = kOffQ + sa((size_t)kStaticMaxKvHeads * 256 * 128);
 constexpr size_t kOffU = kOffAo + sa((size_t)2 * kStaticRows * kStaticMaxQDim * 2);
 constexpr size_t kOffBest = kOffU + sa((size_t)2 * kStaticRows * kStaticMaxFfn * 2);
 constexpr size_t kOffRope = kOffBest + sa((size_t)kStaticRows * 8);
@@ -763,10 +781,10 @@ constexpr size_t kOffWs = kOffSs + sa((size_t)(kStaticMaxHidden / 128) * kStatic
 constexpr size_t kOffCnt = kOffWs + sa((size_t)kStaticMaxSms * 2 * 16 * 128 * 4);
 constexpr size_t kOffAttnO = kOffCnt + sa((size_t)(kStaticMaxVocab / 128 + 64) * 4);
 constexpr size_t kOffAttnMl =
-    kOffAttnO + sa((size_t)kStaticMaxKvHeads * kStaticParts * kStaticMaxGroup * 128 * 4);
+    kOffAttnO + sa((size_t)kStaticMaxKvHeads * kStaticChunks * 64 * 128 * 4);
 constexpr size_t kStaticMaxQkvTiles = (kStaticMaxQDim + 2 * kStaticMaxKvHeads * 128) / 128;
-constexpr size_t kOffQkvPart =
-    kOffAttnMl + sa((size_t)kStaticMaxKvHeads * kStaticParts * kStaticMaxGroup * 8);
+constexpr size_t kOffAttnCnt = kOffAttnMl + sa((size_t)kStaticMaxKvHeads * kStaticChunks * 64 * 8);
+constexpr size_t kOffQkvPart = kOffAttnCnt + sa((size_t)kStaticMaxKvHeads * 8 * 4);
 constexpr size_t kOffQkvRinv = kOffQkvPart + sa(kStaticMaxQkvTiles * 8 * kStaticRows * 128 * 4);
 constexpr size_t kStaticScratchBytes = kOffQkvRinv + sa((size_t)kStaticRows * 4);
 
@@ -854,7 +872,7 @@ extern "C" as2d_status as2d_decode_step_static(as2d_model* mh, void* k_cache, vo
   s.nb_max = 16;
   s.h = (float*)(b + kOffH);
   s.xn = (bf16*)(b + kOffXn);
-  s.q = (float*)(b + kOffQ);
+  s.qimg = (uint8_t*)(b + kOffQ);
   s.ao = (bf16*)(b + kOffAo);
   s.u = (bf16*)(b + kOffU);
   s.best = (unsigned long long*)(b + kOffBest);
@@ -864,11 +882,16 @@ extern "C" as2d_status as2d_decode_step_static(as2d_model* mh, void* k_cache, vo
   s.counters = (int*)(b + kOffCnt);
   s.attn_o = (float*)(b + kOffAttnO);
   s.attn_ml = (float2*)(b + kOffAttnMl);
+  s.attn_cnt = (int*)(b + kOffAttnCnt);
+  s.n_attn_cnt = c.n_kv_heads * 8;
   s.qkv_part = (float*)(b + kOffQkvPart);
   s.qkv_rinv = (float*)(b + kOffQkvRinv);
   s.qkv_split = qkv_split_for(m);
-  s.attn_parts = (capacity + 63) / 64;
-  s.attn_qmax = ((c.n_q_heads / c.n_kv_heads) + 15) / 16 * 16;
+  s.attn_qt = 1;
+  s.attn_chunks = attn_chunks(capacity);
+  if (!encode_cache_map(&s.tm_kc, k_cache, c.head_dim, capacity, (int64_t)c.n_layers * c.n_kv_heads) ||
+      !encode_cache_map(&s.tm_vc, v_cache, c.head_dim, capacity, (int64_t)c.n_layers * c.n_kv_heads))
+    return fail(AS2D_ERR_CUDA, "cuTensorMapEncodeTiled failed for a cache");
   s.tm_xn[0] = sd.tm_xn;
   s.tm_ao[0] = sd.tm_ao;
   s.tm_u[0] = sd.tm_u;
@@ -881,6 +904,7 @@ extern "C" as2d_status as2d_decode_step_static(as2d_model* mh, void* k_cache, vo
   CUDA_TRY(cudaMemsetAsync(b + kOffErr, 0, 256, st));
   CUDA_TRY(cudaMemsetAsync(b + kOffBest, 0, kStaticRows * 8, st));
   CUDA_TRY(cudaMemsetAsync(b + kOffCnt, 0, (size_t)s.n_counters * 4, st));
+  CUDA_TRY(cudaMemsetAsync(b + kOffAttnCnt, 0, (size_t)s.n_attn_cnt * 4, st));
 
   RowMap rm;
   rm.batch = 1;
@@ -893,16 +917,6 @@ extern "C" as2d_status as2d_decode_step_static(as2d_model* mh, void* k_cache, vo
   TcParams tp{};
   tp.h = s.h;
   tp.u = s.u;
-  tp.q = s.q;
-  tp.kc = s.k_cache;
-  tp.vc = s.v_cache;
-  tp.rope = s.rope;
-  tp.len = s.d_len;
-  tp.batch = 1;
-  tp.cap = capacity;
-  tp.nq = c.n_q_heads;
-  tp.nkv = c.n_kv_heads;
-  tp.d = c.head_dim;
   tp.logits = logits;
   tp.best = s.best;
   tp.xn = s.xn;
@@ -913,11 +927,12 @@ extern "C" as2d_status as2d_decode_step_static(as2d_model* mh, void* k_cache, vo
   tp.eps = c.rms_eps;
   tp.hidden = c.hidden;
   for (int l = 0; l < c.n_layers; ++l) {
-    tp.layer = l;
     LAUNCH(AS2D_KERNEL_QKV, tc_project(TC_PART, m, s, rm, m.w_qkv[l], s.tm_xn, m.qkv_rows, H, tp, st));
     LAUNCH(AS2D_KERNEL_ATTENTION, launch_attention_split(rm, m, s, l, st));
     tp.g_next = m.mlp_norm[l];
+    tp.small_ring = 1;
     LAUNCH(AS2D_KERNEL_O, tc_project(TC_RESID, m, s, rm, m.w_o[l], s.tm_ao, H, m.q_dim, tp, st));
+    tp.small_ring = 0;
     LAUNCH(AS2D_KERNEL_GATE_UP, tc_project(TC_SWIGLU, m, s, rm, m.w_gu[l], s.tm_xn, 2 * F, H, tp, st));
     tp.g_next = (l + 1 < c.n_layers) ? m.attn_norm[l + 1] : m.final_norm;
     LAUNCH(AS2D_KERNEL_DOWN, tc_project(TC_RESID, m, s, rm, m.w_down[l], s.tm_u, H, F, tp, st));
@@ -932,4 +947,4 @@ extern "C" as2d_status as2d_decode_step_static(as2d_model* mh, void* k_cache, vo
 
 static_assert(kStaticMaxVocab / 128 + 64 >= (2 * kStaticMaxFfn) / 128 + 64,
               "the counter region covers the largest projection's tiles");
-static_assert(kStaticScratchBytes == 12930048, "as2d.h states the fixed working-memory size");
+static_assert(kStaticScratchBytes == 9735424, "as2d.h states the fixed working-memory size");

@@ -66,6 +66,9 @@ struct TcParams {
   int grid;              // CTAs
   int split;             // TC_PART: CTAs per tile (K split), else 0 (stream-K)
   int defer;             // stream-K: split tiles are finished by tc_reduce_kernel
+  int small_ring;        // a 5-deep ring (token rows <= 16), so that the CTA fits
+                         // on an SM beside an attention CTA and its first weight
+                         // tiles stream while the attention still runs
   float* part;           // TC_PART: [tile][split][part_ld][128] fp32 sums
   float* part_rinv;      // TC_PART: [part_ld] 1 / rms of each token row
   int part_ld;           // rows_alloc
@@ -78,12 +81,6 @@ struct TcParams {
   // epilogue operands
   float* h;              // RESID: h[m][n] += D (ld = N)
   bf16* u;               // SWIGLU: u[m][j], ld = N / 2
-  float* q;              // QKV: rotated queries [m][nq * d]
-  bf16* kc;
-  bf16* vc;
-  const float2* rope;    // [m][d / 2] (cos, sin) of the row's position
-  const int32_t* len;
-  int layer, batch, cap, nq, nkv, d;
   float* logits;         // LOGITS (nullable), ld = N
   unsigned long long* best;
   // RMSNorm folded into the GEMMs: a RESID epilogue leaves, for the next
@@ -166,7 +163,6 @@ struct KvState {
   float* h = nullptr;        // [rows][H] residual stream, fp32
   // bf16 operand buffers hold hi rows [0, rows_alloc) then lo rows
   bf16* xn = nullptr;        // [2 rows][H] next projection's operand bf16(h * g)
-  float* q = nullptr;        // [rows][nq][d] rotated queries
   bf16* ao = nullptr;        // [2 rows][nq d] attention output
   bf16* u = nullptr;         // [2 rows][F] SwiGLU output
   unsigned long long* best = nullptr;  // [rows] packed (logit, index) maxima
@@ -182,12 +178,18 @@ struct KvState {
   int* counters = nullptr;   // [max tiles] stream-K arrival counters
   int n_counters = 0;
   float* ss = nullptr;       // [hidden / 128][rows_alloc] partial sums of h^2
-  float* attn_o = nullptr;   // [batch][n_kv][parts][qmax][d] attention partials
-  float2* attn_ml = nullptr; // [batch][n_kv][parts][qmax] (max, sum) base 2
-  int attn_parts = 0;        // 64-key partitions of the capacity
-  int attn_qmax = 0;         // (kMaxK + 1) * group, rounded up to 16
+  // attention (k_attn.cu): per (request, kv head, 64-query tile)
+  uint8_t* qimg = nullptr;   // query operand images, attn_qimg_bytes(d) each
+  int attn_qt = 0;           // query tiles of the widest request
+  int attn_chunks = 0;       // 1024-key chunks of the capacity
+  float* attn_o = nullptr;   // [batch][n_kv][qt][chunks][64][d] chunk partials
+  float2* attn_ml = nullptr; // [batch][n_kv][qt][chunks][64] (max, sum) base 2
+  int* attn_cnt = nullptr;   // [batch][n_kv][qt][8] chunks arrived per 8-row group; zero between launches
+  int n_attn_cnt = 0;
   // TMA descriptors of the activation operands, per token-row padding
   CUtensorMap tm_xn[kNbCount], tm_ao[kNbCount], tm_u[kNbCount];
+  // TMA descriptors of the caches: [n_layers * batch * n_kv][capacity][d]
+  CUtensorMap tm_kc, tm_vc;
   // measurement support
   int prof_class = -1;
   std::vector<cudaEvent_t> prof_events;  // pairs
@@ -225,8 +227,15 @@ size_t packed_elems(int n_rows, int K);
 cudaError_t pack_weights(bf16* dst, int n_rows, int K, const void* const* segs,
                          const int* seg_rows, int nseg, bool interleave, cudaStream_t st);
 
-// Split-KV attention on the tensor cores + partition merge (k_attn.cu).
-int attn_partitions(int capacity);
+// Attention on the tensor cores (k_attn.cu): query tiles of a request of
+// `rows` rows, 1024-key chunks of a capacity, bytes of one query image.
+int attn_q_tiles(int rows_per_request, int group);
+int attn_chunks(int capacity);
+size_t attn_qimg_bytes(int head_dim);
+// The cache [n_layers][batch][n_kv][capacity][head_dim] bf16 as the 3D tensor
+// map the attention kernel loads key/value tiles through.
+bool encode_cache_map(CUtensorMap* map, const void* cache, int head_dim, int capacity,
+                      int64_t heads);
 cudaError_t launch_attention_split(const RowMap& m, const Model& md, KvState& kv, int layer,
                                    cudaStream_t st);
 

@@ -1,253 +1,647 @@
 // k_attn.cu -- grouped-query attention of a verification block over the
-// retained prefix, split over the key axis (flash-decode), with the causal
-// mask inside the block.
+// retained prefix (Section 3.2: one causal pass over the root and the
+// candidates; App. C.4: rows attend to the committed prefix and to the
+// block's own earlier rows).
 //
-// Row i of request b sits at position L_b + i and attends to keys [0, L_b + i]:
-// the prefilled audio/instruction prefix, the committed tokens, and the
-// block's own rows up to itself.  All G = n_q / n_kv query heads of a key/value
-// head, for all k + 1 rows, form one query matrix of (k + 1) * G rows, so each
-// key/value entry is read from HBM once per block.
+// Row i of request b sits at position L_b + i and attends to keys [0, L_b + i].
+// All G = n_q / n_kv query heads of a key/value head, for all rows of the
+// request, form one query matrix of M * G rows, so each key/value entry is
+// read from HBM once per block (twice when a request has more than 64 query
+// rows, the second time from L2).
 //
-// Pass 0 (qkv_finish_kernel): the QKV projection arrives as split-K partial
-// sums (TC_PART); one CTA per (token row, head) adds them in rank order,
-// scales by the row's 1 / rms, rotates (RoPE) and writes the queries, and
-// appends the new keys and values to the cache.
-// Pass 1 (attn_part_kernel): one CTA per (64-key partition, kv head, request).
-// Keys and values are staged in shared memory -- those already in the cache
-// before the kernel waits for pass 0, the block's own after; each warp takes
-// 16 query rows at a time (4 to 8 warps, by the largest request);
-// S = Q K^T and O = P V run on the tensor cores (mma.sync m16n8k16, bf16 in,
-// fp32 accumulate), with Q and P each split into bf16 hi + lo parts (two MMAs)
-// so that only the bf16 cache itself limits precision; the softmax runs in
-// fp32 in base 2.  Partition boundaries
-// are fixed multiples of 64 positions, so a query's partial results do not
-// depend on the other rows of the call (batch invariance).
-// Pass 2 (attn_merge_kernel): per (row, query head) the partitions' (max,
-// sum, unnormalised output) are combined (log-sum-exp) in an order fixed by
-// the row's own number of partitions.
-#include "attn_dev.cuh"
+// qkv_finish_kernel: the QKV projection arrives as split-K partial sums
+// (TC_PART); one CTA per (token row, head) adds them in rank order, scales by
+// the row's 1 / rms and rotates (RoPE).  Keys and values are appended to the
+// cache; queries, scaled by log2(e) / sqrt(d), are written as bf16 hi and lo
+// parts straight into the tensor-core operand image of their (request, kv
+// head, 64-query tile): 128 rows (row 2q the hi part of query q, row 2q + 1
+// its lo part) of d elements in the 128-byte-swizzled K-major layout, one
+// 16 KB region per 64 columns.
+//
+// attn_tc_kernel: one CTA per 128-key tile of one (request, kv head, query
+// tile); a cluster of 8 CTAs covers one chunk of 1024 keys.  Per CTA:
+//   * the tile's keys and values arrive by TMA (3D map over the cache, 128-
+//     byte swizzle; tiles holding only entries older than this call are
+//     requested before the wait for the finishing kernel), the query image
+//     by one bulk copy;
+//   * S = Q K^T on tcgen05 (M = 128: the hi and lo rows of 64 queries
+//     interleaved, N = 128 keys) into TMEM; thread t reads lane t, so each
+//     query's hi and lo scores sit in adjacent lanes of one warp and are
+//     added by a shuffle, each lane keeping half of the keys; masking (causal,
+//     and keys past the call's end) and P = 2^(S - m) with the tile's own
+//     maximum m and sum l;
+//   * O = P V on tcgen05 (P's hi and lo rows interleaved the same way; B = V
+//     read MN-major from the TMA image); hi + lo added by a shuffle, each lane
+//     keeping half of the dims;
+//   * the tile partials (m, l, O) are pushed through distributed shared
+//     memory to the CTA that folds their query rows (CTA r: rows 8r..8r+7),
+//     which folds the cluster's 8 tiles in tile order.  With one chunk the
+//     result is normalised and written (bf16 hi, lo); otherwise the CTA's rows
+//     of the chunk partial go to memory and the last CTA of those rows to
+//     arrive, over the chunks of the (request, kv head, query tile), folds
+//     them in chunk order.
+// Every fold boundary is a fixed absolute key position (128-key tiles,
+// 1024-key chunks), and a fold with a part a row cannot see (fully masked:
+// m = -inf, l = 0, O = 0) leaves it bitwise unchanged, so a row's result does
+// not depend on the other rows of the call (batch invariance).
+#include "as2d_internal.h"
+#include "ptx_sm100.cuh"
 
 namespace as2d {
 namespace {
 
-using namespace attn;
+constexpr int kTile = 128;    // keys per CTA
+constexpr int kCluster = 8;   // CTAs per cluster
+constexpr int kChunk = kTile * kCluster;
+constexpr int kQT = 64;       // queries per query tile (hi and lo rows interleaved)
+constexpr uint32_t kRegion = 128 * 128;  // one 64-column region of 128 rows, bytes
+constexpr uint32_t kSmemAttn = 3 * 32768 + 64 * 8 + 8 * 4 + 4 * 8 + 16 + 1024;
 
-template <int D>
-__global__ void __launch_bounds__(256, 1) attn_part_kernel(AttnArgs a) {
-  __shared__ __align__(16) bf16 sK[kPart][kPitch];
-  __shared__ __align__(16) bf16 sV[kPart][kPitch];
-  // item blockIdx.x -> (request, partition): only each request's own partitions
-  int b = 0;
-  while (b + 1 < a.batch && a.part_start[b + 1] <= (int)blockIdx.x) ++b;
-  const int part = (int)blockIdx.x - a.part_start[b];
-  const bool fits = rows_fit(a.len[b], a.rm.start[b + 1] - a.rm.start[b], a.cap);
-  // the keys/values already in the cache do not depend on the predecessor
-  if (fits) stage_old_kv<D>(a, a.layer, part, blockIdx.y, b, sK, sV, threadIdx.x, blockDim.x);
-  ptx::griddep_wait();
-  ptx::griddep_launch_dependents();
-  if (!fits) return;  // flagged by the embedding kernel; nothing of the cache is read
-  part_item<D, true>(a, a.layer, part, blockIdx.y, b, sK, sV, threadIdx.x, blockDim.x, 0);
+struct AttnArgs {
+  RowMap rm;
+  const int32_t* len;
+  int layer, batch, cap, nq, nkv;
+  float qscale;  // log2(e) / sqrt(d), folded into the stored queries
+  // split-K sums of the QKV projection (TC_PART)
+  const float* qkv_part;  // [tile][split][qkv_ld][128], tile = column / 128
+  const float* qkv_rinv;  // [qkv_ld] 1 / rms of each token row
+  const float2* rope;     // [rows][d / 2] (cos, sin)
+  int qkv_split, qkv_ld;
+  bf16* kc;
+  bf16* vc;
+  uint8_t* qimg;          // [batch][nkv][qt_max] operand images, 256 d bytes each
+  int qt_max;
+  float* ws_o;            // [batch][nkv][qt_max][chunks_max][64][d] chunk partials
+  float2* ws_ml;          // [batch][nkv][qt_max][chunks_max][64] (max, sum), base 2
+  int chunks_max;
+  int* cnt;               // [batch][nkv][qt_max][8] chunks arrived per 8-row group
+  bf16* ao;               // [2 rows][nq d]: hi rows, then lo rows from lo_row
+  int lo_row;
+  int32_t* err;
+  unsigned long long timeout_ns;
+  // clusters of request b: [cl_start[b], cl_start[b + 1]); n_ch[b] of them per
+  // query tile (chunks covering the host's bound of the request's keys)
+  int32_t cl_start[kMaxBatch + 1];
+  int32_t n_ch[kMaxBatch];
+};
+
+// ---- finishing the QKV projection from its split-K sums ----------------------
+
+// Projection value of column col (q, k or v head * D + e) for token row gm:
+// the split parts added in rank order, times the row's 1 / rms.
+__device__ __forceinline__ float qkv_value(const AttnArgs& a, int col, int gm) {
+  const float* src = a.qkv_part + ((size_t)(col >> 7) * a.qkv_split * a.qkv_ld + gm) * 128 + (col & 127);
+  float v[8];
+#pragma unroll
+  for (int r = 0; r < 8; ++r) v[r] = r < a.qkv_split ? src[(size_t)r * a.qkv_ld * 128] : 0.f;
+  float acc = 0.f;
+#pragma unroll
+  for (int r = 0; r < 8; ++r)
+    if (r < a.qkv_split) acc += v[r];
+  return acc * a.qkv_rinv[gm];
 }
 
-// The QKV projection finished from its split-K sums (TC_PART): one CTA of
-// D / 2 threads per (token row, head); thread e
-// forms the pair (e, e + D/2) -- rotated queries into q, rotated keys and
-// values appended to the cache.  Every load of a thread is issued before the
-// first is used.
+// Byte offset of element (row r, column e) in a 128-row operand image of
+// 128-byte-swizzled K-major bf16: 64-column regions of kRegion bytes, 16-byte
+// chunk j of row r stored at chunk j ^ (r mod 8).
+__device__ __forceinline__ uint32_t img_off(int r, int e) {
+  const int reg = e >> 6, j = (e & 63) >> 3;
+  return (uint32_t)reg * kRegion + (uint32_t)r * 128u + (uint32_t)((j ^ (r & 7)) << 4) +
+         (uint32_t)((e & 7) << 1);
+}
+
+// One CTA of D / 2 threads per (token row, head); thread e forms the pair
+// (e, e + D/2).  Rotate-half RoPE: x' = x cos - x_p sin at e, x_p cos + x sin
+// at e + D/2.
 template <int D>
 __global__ void __launch_bounds__(D / 2) qkv_finish_kernel(AttnArgs a) {
   ptx::griddep_wait();
   ptx::griddep_launch_dependents();
   constexpr int H2 = D / 2;
   const int gm = blockIdx.x, head = blockIdx.y, e = threadIdx.x;
-  const int b = row_request(a.rm, gm), pos = a.len[b] + (gm - a.rm.start[b]);
-  if (!rows_fit(a.len[b], a.rm.start[b + 1] - a.rm.start[b], a.cap)) return;  // no append
-  const float2 y = (head < a.nq + a.nkv) ? qk_rotated<D>(a, head, e, gm)
-                                         : make_float2(qkv_value(a, head * D + e, gm),
-                                                       qkv_value(a, head * D + e + H2, gm));
+  const int b = row_request(a.rm, gm), i = gm - a.rm.start[b];
+  if (!rows_fit(a.len[b], a.rm.start[b + 1] - a.rm.start[b], a.cap)) return;  // flagged
+  const int pos = a.len[b] + i;
+  float y0, y1;
+  const float x = qkv_value(a, head * D + e, gm), xp = qkv_value(a, head * D + e + H2, gm);
+  if (head < a.nq + a.nkv) {
+    const float2 cs = a.rope[(size_t)gm * H2 + e];
+    y0 = fmaf(x, cs.x, -(xp * cs.y));
+    y1 = fmaf(xp, cs.x, x * cs.y);
+  } else {
+    y0 = x;
+    y1 = xp;
+  }
   if (head < a.nq) {
-    float* q = const_cast<float*>(a.q) + (size_t)gm * a.nq * D + head * D;
-    q[e] = y.x;
-    q[e + H2] = y.y;
+    const int G = a.nq / a.nkv, g = head / G;
+    const int qg = i * G + (head - g * G);
+    const int qt = qg / kQT, q = qg - qt * kQT;
+    uint8_t* img = a.qimg + ((size_t)(b * a.nkv + g) * a.qt_max + qt) * (size_t)(256 * D);
+    const float v0 = y0 * a.qscale, v1 = y1 * a.qscale;
+    const bf16 h0 = __float2bfloat16_rn(v0), h1 = __float2bfloat16_rn(v1);
+    *reinterpret_cast<bf16*>(img + img_off(2 * q, e)) = h0;
+    *reinterpret_cast<bf16*>(img + img_off(2 * q, e + H2)) = h1;
+    *reinterpret_cast<bf16*>(img + img_off(2 * q + 1, e)) =
+        __float2bfloat16_rn(v0 - __bfloat162float(h0));
+    *reinterpret_cast<bf16*>(img + img_off(2 * q + 1, e + H2)) =
+        __float2bfloat16_rn(v1 - __bfloat162float(h1));
   } else {
     const bool is_k = head < a.nq + a.nkv;
     const int g = is_k ? head - a.nq : head - a.nq - a.nkv;
-    bf16* dst = const_cast<bf16*>(is_k ? a.kc : a.vc) +
-                ((((size_t)a.layer * a.batch + b) * a.nkv + g) * a.cap + pos) * D;
-    dst[e] = __float2bfloat16_rn(y.x);
-    dst[e + H2] = __float2bfloat16_rn(y.y);
+    bf16* dst = (is_k ? a.kc : a.vc) + ((((size_t)a.layer * a.batch + b) * a.nkv + g) * a.cap + pos) * D;
+    dst[e] = __float2bfloat16_rn(y0);
+    dst[e + H2] = __float2bfloat16_rn(y1);
   }
 }
 
-// Pass 2 for one (row, query head) per CTA of D x (1..4) threads.  All the
-// partitions' (max, sum) pairs are loaded together into shared memory; the
-// maximum, the weights 2^(m_p - M) and the total (warp 0: lane e adds
-// partitions e, e + 32, ... in order, then a butterfly) follow; the outputs
-// are added by gs = min(4, ceil(parts / 32)) groups of D threads, group q
-// taking a contiguous run of partitions in order, 32 loads in flight, and the
-// groups' sums are added in group order.  Every order depends on the row's
-// own number of partitions alone; with at most 32 partitions (positions below
-// 2048) it is the single in-order sum.
-constexpr int kMergeGroups = 4;
+// ---- attention over 128-key tiles on the tensor cores ------------------------
+
+// 2^x on the special-function unit (ftz: results below 2^-126 are 0).
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// Values x[0..7] of columns e0..e0+7 (e0 % 8 == 0) of query q, as bf16 hi
+// parts into row 2q and lo parts (x - hi) into row 2q + 1 of an operand image.
+__device__ __forceinline__ void put_hilo8(uint8_t* img, int q, int e0, const float* x) {
+  uint32_t hw[4], lw[4];
+#pragma unroll
+  for (int u = 0; u < 4; ++u) {
+    const __nv_bfloat162 hv = __floats2bfloat162_rn(x[2 * u], x[2 * u + 1]);
+    const float2 hf = __bfloat1622float2(hv);
+    const __nv_bfloat162 lv = __floats2bfloat162_rn(x[2 * u] - hf.x, x[2 * u + 1] - hf.y);
+    hw[u] = *reinterpret_cast<const uint32_t*>(&hv);
+    lw[u] = *reinterpret_cast<const uint32_t*>(&lv);
+  }
+  *reinterpret_cast<uint4*>(img + img_off(2 * q, e0)) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+  *reinterpret_cast<uint4*>(img + img_off(2 * q + 1, e0)) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+}
+
+__device__ __forceinline__ void dsmem_st_f4(uint32_t addr, float4 v) {
+  asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "f"(v.x), "f"(v.y),
+               "f"(v.z), "f"(v.w)
+               : "memory");
+}
+
+__device__ __forceinline__ void dsmem_st_f2(uint32_t addr, float2 v) {
+  asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(addr), "f"(v.x), "f"(v.y)
+               : "memory");
+}
+
+// 64 columns of this thread's TMEM lane starting at `col`, into v.
+__device__ __forceinline__ void tmem_ld64(uint32_t taddr, float (&v)[64]) {
+  uint32_t a[32], b[32];
+  ptx::tmem_ld32(taddr, a);
+  ptx::tmem_ld32(taddr + 32, b);
+  ptx::tmem_ld_wait();
+#pragma unroll
+  for (int j = 0; j < 32; ++j) {
+    v[j] = __uint_as_float(a[j]);
+    v[32 + j] = __uint_as_float(b[j]);
+  }
+}
+
+// The weight of a part (max m) in a fold whose maximum is M: 2^(m - M), 0
+// where m = -inf (nothing of the part is visible to the row), exactly 1 for
+// the part holding the maximum.  Parts of weight 0 are skipped by the folds,
+// so a part a row cannot see leaves its result bitwise unchanged.
+__device__ __forceinline__ float part_weight(float m, float M) {
+  return m == -INFINITY ? 0.f : (m == M ? 1.f : ex2(m - M));
+}
 
 template <int D>
-__global__ void __launch_bounds__(kMergeGroups * D) attn_merge_kernel(AttnArgs a) {
-  constexpr int PF = 32;
-  __shared__ float2 s_ml[kMaxParts];
-  __shared__ float s_w[kMaxParts];
-  __shared__ float s_red[kMergeGroups * D / 32];
-  __shared__ float s_o[kMergeGroups - 1][D];
-  __shared__ float s_l;
-  ptx::griddep_wait();
-  ptx::griddep_launch_dependents();
-  const int r = blockIdx.x, j = blockIdx.y, tid = threadIdx.x, nthr = blockDim.x;
-  const int G = a.nq / a.nkv;
-  const int b = row_request(a.rm, r);
-  const int i = r - a.rm.start[b];
-  const int g = j / G, qr = i * G + (j - g * G);
-  if (!rows_fit(a.len[b], a.rm.start[b + 1] - a.rm.start[b], a.cap)) {
-    // a skipped request: zero output, no partition is read
-    for (int e = tid; e < D; e += nthr) {
-      a.ao[(size_t)r * a.nq * D + (size_t)j * D + e] = __float2bfloat16_rn(0.f);
-      a.ao[(size_t)(a.lo_row + r) * a.nq * D + (size_t)j * D + e] = __float2bfloat16_rn(0.f);
+__global__ void __launch_bounds__(128, 2)
+    attn_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
+                   const __grid_constant__ AttnArgs a) {
+  constexpr int NR = D / 64;          // 64-column regions of a K / V tile
+  constexpr uint32_t KV_BYTES = 2u * NR * kRegion;
+  constexpr uint32_t Q_BYTES = 2u * kQT * D * 2;
+  constexpr int DH = D / 2;           // dims each thread of a hi/lo pair keeps
+  constexpr int DT = D / 16;          // dims per thread in the folds (8 rows x 16 threads)
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* sm = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  uint8_t* R0 = sm;            // Q image -> P image -> the partials received from the cluster
+  uint8_t* R1 = sm + 32768;    // K tile
+  uint8_t* R2 = sm + 65536;    // V tile
+  float2* s_rml = reinterpret_cast<float2*>(sm + 98304);  // [8 tiles][8 rows] received (max, sum)
+  float* s_x = reinterpret_cast<float*>(s_rml + 64);      // [8] scratch
+  uint64_t* bars = reinterpret_cast<uint64_t*>(s_x + 8);  // q, kv, mma1, mma2
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 4);
+  int* s_flag = reinterpret_cast<int*>(tslot + 1);
+
+  const int tid = threadIdx.x, warp = tid >> 5;
+  const uint32_t rank = ptx::cluster_rank();
+  const int cl = (int)(blockIdx.x / kCluster), g = blockIdx.y;
+  int b = 0;
+  while (b + 1 < a.rm.batch && a.cl_start[b + 1] <= cl) ++b;
+  const int ci = cl - a.cl_start[b];
+  const int qt = ci / a.n_ch[b], c = ci - qt * a.n_ch[b];
+  const int t = c * kCluster + (int)rank, p0 = t * kTile;
+  const int r0 = a.rm.start[b], M = a.rm.start[b + 1] - r0;
+  const int G = a.nq / a.nkv, qn = M * G;
+  const int L = a.len[b];
+  const bool fits = rows_fit(L, M, a.cap);
+  const int kend = L + M;
+  const int n_tiles = fits ? (kend + kTile - 1) / kTile : 0;
+  const int n_chunks = (n_tiles + kCluster - 1) / kCluster;
+  const bool active = t < n_tiles;      // this CTA's tile holds keys
+  const bool cl_active = c < n_chunks;  // uniform over the cluster
+  const int z = (a.layer * a.batch + b) * a.nkv + g;
+  const uint8_t* qsrc = a.qimg + ((size_t)(b * a.nkv + g) * a.qt_max + qt) * (size_t)Q_BYTES;
+
+  if (tid == 0) {
+    for (int i = 0; i < 4; ++i) ptx::mbar_init(&bars[i], 1);
+    ptx::fence_mbar_init();
+  }
+  if (warp == 0) ptx::tmem_alloc(tslot, 256);
+  ptx::tc_fence_before();
+  __syncthreads();
+  ptx::tc_fence_after();
+  const uint32_t tmem = *tslot;
+  const uint32_t lane_base = (uint32_t)(32 * warp) << 16;
+
+  // a tile of entries older than this call does not depend on the finishing
+  // kernel: request it before the wait
+  const bool early = active && p0 + kTile <= L;
+  const uint64_t pol = ptx::policy_evict_first();
+  auto load_kv = [&]() {
+    ptx::mbar_arrive_expect_tx(&bars[1], KV_BYTES);
+#pragma unroll
+    for (int h = 0; h < NR; ++h) {
+      ptx::tma_load_3d(R1 + h * kRegion, &tmK, &bars[1], 64 * h, p0, z, pol);
+      ptx::tma_load_3d(R2 + h * kRegion, &tmV, &bars[1], 64 * h, p0, z, pol);
     }
+  };
+  if (tid == 0 && early) {
+    ptx::prefetch_tmap(&tmK);
+    ptx::prefetch_tmap(&tmV);
+    load_kv();
+  }
+  ptx::griddep_wait();
+  // every CTA of this grid holds its TMEM by now: the next kernel (the O
+  // projection) may start and stream its first weight tiles meanwhile
+  ptx::griddep_launch_dependents();
+  if (tid == 0 && active) {
+    if (!early) load_kv();
+    ptx::mbar_arrive_expect_tx(&bars[0], Q_BYTES);
+    ptx::bulk_load(R0, qsrc, Q_BYTES, &bars[0], ptx::policy_evict_last());
+  }
+
+  // Thread tid reads TMEM lane tid: query q = tid / 2, its hi part (pt = 0)
+  // or lo part (pt = 1).  After the exchange with its partner lane it keeps
+  // keys [64 pt, 64 pt + 64) of S and dims [DH pt, DH pt + DH) of O.
+  const int q = tid >> 1, pt = tid & 1;
+  const int qg = qt * kQT + q;
+  const int lim = qg < qn ? L + qg / G : -1;  // the query's last visible key
+  float m = -INFINITY, l = 0.f;               // the tile partial of query q
+  float o[DH];
+#pragma unroll
+  for (int j = 0; j < DH; ++j) o[j] = 0.f;
+  bool ok = true;
+  if (active) {
+    ok = ptx::mbar_wait(&bars[0], 0, a.timeout_ns) && ptx::mbar_wait(&bars[1], 0, a.timeout_ns);
+    ok = ptx::group_all(ok, 1, 128);
+    if (!ok) {
+      if (tid == 0) {
+        atomicOr(a.err, kErrTimeout);
+        // the copies may still be in flight: wait for them before the CTA ends
+        ptx::mbar_wait(&bars[0], 0, a.timeout_ns);
+        ptx::mbar_wait(&bars[1], 0, a.timeout_ns);
+      }
+      __syncthreads();
+    }
+  }
+  if (active && ok) {
+    if (tid == 0) {
+      ptx::tc_fence_after();
+      constexpr uint32_t IDESC1 = ptx::idesc_bf16_f32(128, kTile);
+#pragma unroll
+      for (int kk = 0; kk < D / 16; ++kk) {
+        const uint64_t ad = ptx::sdesc_sw128(ptx::smem_u32(R0 + (kk >> 2) * kRegion)) + 2 * (kk & 3);
+        const uint64_t bd = ptx::sdesc_sw128(ptx::smem_u32(R1 + (kk >> 2) * kRegion)) + 2 * (kk & 3);
+        ptx::mma_bf16(tmem, ad, bd, IDESC1, kk > 0 ? 1u : 0u);
+      }
+      ptx::mma_commit(&bars[2]);
+    }
+    // values past the call's last key (stale entries, or NaN in a poisoned
+    // cache) would reach O through 0 * V: zero those rows of the V tile
+    // while the first product runs
+    const int z0 = kend - p0;
+    if (z0 < kTile) {
+      for (int idx = tid; idx < (kTile - z0) * NR * 8; idx += 128) {
+        const int r = z0 + idx / (NR * 8), rest = idx - (idx / (NR * 8)) * (NR * 8);
+        *reinterpret_cast<uint4*>(R2 + (rest >> 3) * kRegion + r * 128 + (rest & 7) * 16) =
+            make_uint4(0, 0, 0, 0);
+      }
+      ptx::fence_proxy_async_smem();
+    }
+    const bool ok1 = ptx::group_all(ptx::mbar_wait(&bars[2], 0, a.timeout_ns), 1, 128);
+    ptx::tc_fence_after();
+    bool ok2 = ok1;
+    if (ok1) {
+      // S = hi + lo of this thread's keys, masked; the tile's maximum and
+      // P = 2^(S - m) with the partner lane
+      float sv[64];
+      {
+        float v0[64], v1[64];
+        tmem_ld64(tmem + lane_base, v0);
+        tmem_ld64(tmem + lane_base + 64, v1);
+#pragma unroll
+        for (int j = 0; j < 64; ++j) {
+          const float mine = pt ? v1[j] : v0[j], other = pt ? v0[j] : v1[j];
+          sv[j] = mine + __shfl_xor_sync(0xFFFFFFFFu, other, 1);
+        }
+      }
+      const int kb = p0 + 64 * pt;
+      float mx = -INFINITY;
+#pragma unroll
+      for (int j = 0; j < 64; ++j)
+        if (kb + j <= lim) mx = fmaxf(mx, sv[j]);
+      m = fmaxf(mx, __shfl_xor_sync(0xFFFFFFFFu, mx, 1));
+      float ls = 0.f;
+#pragma unroll
+      for (int j = 0; j < 64; ++j) {
+        sv[j] = (kb + j <= lim) ? ex2(sv[j] - m) : 0.f;
+        ls += sv[j];
+      }
+      const float lo_ = __shfl_xor_sync(0xFFFFFFFFu, ls, 1);
+      l = pt ? lo_ + ls : ls + lo_;  // keys 0..63, then 64..127
+      // P as bf16 hi (row 2q) and lo (row 2q + 1) parts, K-major by key
+#pragma unroll
+      for (int ch = 0; ch < 8; ++ch) put_hilo8(R0, q, 64 * pt + 8 * ch, sv + 8 * ch);
+      ptx::fence_proxy_async_smem();
+      __syncthreads();
+      if (tid == 0) {
+        ptx::tc_fence_after();
+        constexpr uint32_t IDESC2 = ptx::idesc_bf16_f32(128, D, true);
+#pragma unroll
+        for (int kk = 0; kk < kTile / 16; ++kk) {
+          const uint64_t ad = ptx::sdesc_sw128(ptx::smem_u32(R0 + (kk >> 2) * kRegion)) + 2 * (kk & 3);
+          const uint64_t bd = ptx::sdesc_sw128_mn(ptx::smem_u32(R2) + kk * 2048u, kRegion, 1024u);
+          ptx::mma_bf16(tmem + 128, ad, bd, IDESC2, kk > 0 ? 1u : 0u);
+        }
+        ptx::mma_commit(&bars[3]);
+      }
+      ok2 = ptx::group_all(ptx::mbar_wait(&bars[3], 0, a.timeout_ns), 1, 128);
+      ptx::tc_fence_after();
+      if (ok2) {
+        // O = hi + lo of this thread's dims
+#pragma unroll
+        for (int c0 = 0; c0 < D; c0 += 64) {
+          float v[64];
+          tmem_ld64(tmem + lane_base + 128 + c0, v);
+#pragma unroll
+          for (int j = 0; j < 64; ++j) {
+            const int d = c0 + j;  // compile-time after unrolling
+            const bool mine = (d / DH) == pt;
+            const float x = __shfl_xor_sync(0xFFFFFFFFu, v[j], 1);
+            if (mine) o[d - pt * DH] = v[j] + x;
+          }
+        }
+      }
+    }
+    if (!(ok1 && ok2)) {
+      if (tid == 0) {
+        atomicOr(a.err, kErrTimeout);
+        // no MMA may still run when TMEM is freed
+        ptx::mbar_wait(&bars[2], 0, a.timeout_ns);
+        if (ok1) ptx::mbar_wait(&bars[3], 0, a.timeout_ns);
+      }
+      m = -INFINITY;  // nothing of this tile is passed on
+    }
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  if (warp == 0) ptx::tmem_dealloc(tmem, 256);
+  if (!cl_active) return;  // the whole cluster holds no keys of this request
+
+  // ---- the cluster's tile partials, pushed to the CTA that folds them ----
+  // CTA r folds query rows 8r..8r+7; it receives, from every CTA i of the
+  // cluster, rows (max, sum) into s_rml[i][row] and O into its R0 as
+  // [i][row][d] (every CTA's P image is consumed once all pass this barrier)
+  ptx::cluster_sync();
+  if (active) {
+    const uint32_t dst_rank = (uint32_t)(q >> 3), row = (uint32_t)(q & 7);
+    if (pt == 0)
+      dsmem_st_f2(ptx::dsmem_map(ptx::smem_u32(s_rml + rank * 8 + row), dst_rank), make_float2(m, l));
+    if (m != -INFINITY) {
+      const uint32_t dst = ptx::dsmem_map(
+          ptx::smem_u32(reinterpret_cast<float*>(R0) + (rank * 8 + row) * D + pt * DH), dst_rank);
+#pragma unroll
+      for (int u = 0; u < DH / 4; ++u)
+        dsmem_st_f4(dst + 16u * u, make_float4(o[4 * u], o[4 * u + 1], o[4 * u + 2], o[4 * u + 3]));
+    }
+  }
+  ptx::cluster_sync();
+
+  // ---- fold (thread: query row 8 rank + fj, dims [fd, fd + DT)) ----------
+  const int n_here = min(kCluster, n_tiles - c * kCluster);  // tiles of this chunk with keys
+  const int fj = tid >> 4, fr = 8 * (int)rank + fj, fd = DT * (tid & 15);
+  float fm = -INFINITY;
+  float2 pml[kCluster];
+#pragma unroll
+  for (int i = 0; i < kCluster; ++i) {
+    pml[i] = (i < n_here) ? s_rml[i * 8 + fj] : make_float2(-INFINITY, 0.f);
+    fm = fmaxf(fm, pml[i].x);
+  }
+  float fl = 0.f, fo[DT];
+#pragma unroll
+  for (int e = 0; e < DT; ++e) fo[e] = 0.f;
+#pragma unroll
+  for (int i = 0; i < kCluster; ++i) {
+    const float w = part_weight(pml[i].x, fm);
+    if (w != 0.f) {
+      fl += pml[i].y * w;
+      const float4* src = reinterpret_cast<const float4*>(reinterpret_cast<float*>(R0) +
+                                                          (i * 8 + fj) * D + fd);
+#pragma unroll
+      for (int u = 0; u < DT / 4; ++u) {
+        const float4 v = src[u];
+        fo[4 * u + 0] += v.x * w;
+        fo[4 * u + 1] += v.y * w;
+        fo[4 * u + 2] += v.z * w;
+        fo[4 * u + 3] += v.w * w;
+      }
+    }
+  }
+  // normalise and write the row's dims (o / l as bf16 hi, lo)
+  auto write_out = [&](const float* o_, float Ls) {
+    const int fqg = qt * kQT + fr;
+    if (fqg >= qn) return;
+    const int i = fqg / G, hq = g * G + (fqg - i * G);
+    const size_t at = (size_t)(r0 + i) * a.nq * D + (size_t)hq * D + fd;
+    uint32_t hw[DT / 2], lw[DT / 2];
+#pragma unroll
+    for (int e = 0; e < DT / 2; ++e) {
+      const float v0 = o_[2 * e] / Ls, v1 = o_[2 * e + 1] / Ls;
+      const __nv_bfloat162 hv = __floats2bfloat162_rn(v0, v1);
+      const float2 hf = __bfloat1622float2(hv);
+      const __nv_bfloat162 lv = __floats2bfloat162_rn(v0 - hf.x, v1 - hf.y);
+      hw[e] = *reinterpret_cast<const uint32_t*>(&hv);
+      lw[e] = *reinterpret_cast<const uint32_t*>(&lv);
+    }
+#pragma unroll
+    for (int u = 0; u < DT / 8; ++u) {
+      *reinterpret_cast<uint4*>(a.ao + at + 8 * u) =
+          make_uint4(hw[4 * u], hw[4 * u + 1], hw[4 * u + 2], hw[4 * u + 3]);
+      *reinterpret_cast<uint4*>(a.ao + (size_t)a.lo_row * a.nq * D + at + 8 * u) =
+          make_uint4(lw[4 * u], lw[4 * u + 1], lw[4 * u + 2], lw[4 * u + 3]);
+    }
+    if (DT % 8) {  // D = 64: four dims
+      *reinterpret_cast<uint2*>(a.ao + at) = make_uint2(hw[0], hw[1]);
+      *reinterpret_cast<uint2*>(a.ao + (size_t)a.lo_row * a.nq * D + at) = make_uint2(lw[0], lw[1]);
+    }
+  };
+  if (n_chunks == 1) {
+    write_out(fo, fl);
     return;
   }
-  const int pos = a.len[b] + i;
-  const int nparts = pos / kPart + 1;
-  const size_t base = (size_t)(b * a.nkv + g) * a.parts_max * a.qmax + qr;
-  const int want = (nparts + 31) / 32;
-  const int gs = want < kMergeGroups ? want : kMergeGroups;
-  const int chunk = (nparts + gs - 1) / gs;
-  const int grp = tid / D, e = tid - grp * D;
-  const int p_begin = grp * chunk;
-  const int p_end = (p_begin + chunk) < nparts ? (p_begin + chunk) : nparts;
-  // the group's first PF outputs are in flight with the (max, sum) loads
-  float ov[PF];
-  if (grp < gs) {
+  // ---- several chunks: this CTA's rows of the chunk partial go to memory;
+  // the last chunk's CTA of these rows to arrive folds them in chunk order
+  const size_t item = (size_t)(b * a.nkv + g) * a.qt_max + qt;
+  {
+    const size_t pc = item * a.chunks_max + c;
+    float4* dst = reinterpret_cast<float4*>(a.ws_o + (pc * kQT + fr) * D + fd);
 #pragma unroll
-    for (int u = 0; u < PF; ++u)
-      ov[u] = (p_begin + u < p_end) ? a.ws_o[(base + (size_t)(p_begin + u) * a.qmax) * D + e] : 0.f;
-  }
-  for (int p = tid; p < nparts; p += nthr) s_ml[p] = a.ws_ml[base + (size_t)p * a.qmax];
-  __syncthreads();
-  float M = -INFINITY;
-  for (int p = tid; p < nparts; p += nthr) M = fmaxf(M, s_ml[p].x);
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xFFFFFFFFu, M, o));
-  if ((tid & 31) == 0) s_red[tid >> 5] = M;
-  __syncthreads();
-  M = s_red[0];
-  for (int w = 1; w < nthr / 32; ++w) M = fmaxf(M, s_red[w]);
-  for (int p = tid; p < nparts; p += nthr) {
-    const float mp = s_ml[p].x;
-    s_w[p] = (mp == -INFINITY) ? 0.f : exp2f(mp - M);
+    for (int u = 0; u < DT / 4; ++u)
+      dst[u] = make_float4(fo[4 * u], fo[4 * u + 1], fo[4 * u + 2], fo[4 * u + 3]);
+    if ((tid & 15) == 0) a.ws_ml[pc * kQT + fr] = make_float2(fm, fl);
   }
   __syncthreads();
-  if (tid < 32) {
-    float l = 0.f;
-    for (int p = tid; p < nparts; p += 32) l += s_ml[p].y * s_w[p];
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xFFFFFFFFu, l, o);
-    if (tid == 0) s_l = l;
+  int* cnt = a.cnt + item * kCluster + rank;
+  if (tid == 0) {
+    __threadfence();  // the CTA's writes above, before its arrival
+    const int prev = atomicAdd(cnt, 1);
+    const int last = prev == n_chunks - 1;
+    if (last) {
+      *cnt = 0;  // every chunk of these rows has arrived
+      __threadfence();
+    }
+    *s_flag = last;
   }
-  float o = 0.f;
-  if (grp < gs) {
-    for (int p0 = p_begin; p0 < p_end; p0 += PF) {
-      if (p0 > p_begin) {
+  __syncthreads();
+  if (!*s_flag) return;
+  float cm = -INFINITY;
+  for (int cc = 0; cc < n_chunks; ++cc)
+    cm = fmaxf(cm, __ldcg(a.ws_ml + (item * a.chunks_max + cc) * kQT + fr).x);
+  float cl_ = 0.f, co[DT];
 #pragma unroll
-        for (int u = 0; u < PF; ++u)
-          ov[u] = (p0 + u < p_end) ? a.ws_o[(base + (size_t)(p0 + u) * a.qmax) * D + e] : 0.f;
+  for (int e = 0; e < DT; ++e) co[e] = 0.f;
+  for (int c0 = 0; c0 < n_chunks; c0 += 8) {
+    // eight chunks' values in flight at a time
+    float4 v[8][DT / 4];
+    float2 ml[8];
+#pragma unroll
+    for (int u8 = 0; u8 < 8; ++u8)
+      if (c0 + u8 < n_chunks) {
+        const size_t pc = item * a.chunks_max + c0 + u8;
+        ml[u8] = __ldcg(a.ws_ml + pc * kQT + fr);
+        const float4* src = reinterpret_cast<const float4*>(a.ws_o + (pc * kQT + fr) * D + fd);
+#pragma unroll
+        for (int u = 0; u < DT / 4; ++u) v[u8][u] = __ldcg(src + u);
       }
 #pragma unroll
-      for (int u = 0; u < PF; ++u)
-        if (p0 + u < p_end) o += ov[u] * s_w[p0 + u];
-    }
-    if (grp > 0) s_o[grp - 1][e] = o;
+    for (int u8 = 0; u8 < 8; ++u8)
+      if (c0 + u8 < n_chunks) {
+        const float w = part_weight(ml[u8].x, cm);
+        if (w != 0.f) {
+          cl_ += ml[u8].y * w;
+#pragma unroll
+          for (int u = 0; u < DT / 4; ++u) {
+            co[4 * u + 0] += v[u8][u].x * w;
+            co[4 * u + 1] += v[u8][u].y * w;
+            co[4 * u + 2] += v[u8][u].z * w;
+            co[4 * u + 3] += v[u8][u].w * w;
+          }
+        }
+      }
   }
-  __syncthreads();
-  if (grp == 0) {
-    for (int q = 1; q < gs; ++q) o += s_o[q - 1][e];
-    const float ov_ = o / s_l;
-    const bf16 oh = __float2bfloat16_rn(ov_);
-    a.ao[(size_t)r * a.nq * D + (size_t)j * D + e] = oh;
-    a.ao[(size_t)(a.lo_row + r) * a.nq * D + (size_t)j * D + e] =
-        __float2bfloat16_rn(ov_ - __bfloat162float(oh));
-  }
+  write_out(co, cl_);
+}
+
+template <int D>
+cudaError_t launch_attn(const CUtensorMap& tk, const CUtensorMap& tv, const AttnArgs& a,
+                        int clusters, cudaStream_t st) {
+  static const cudaError_t attr = cudaFuncSetAttribute(
+      attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemAttn);
+  if (attr != cudaSuccess) return attr;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(clusters * kCluster, a.nkv);
+  cfg.blockDim = dim3(128);
+  cfg.dynamicSmemBytes = kSmemAttn;
+  cfg.stream = st;
+  cudaLaunchAttribute attr2[2];
+  attr2[0].id = cudaLaunchAttributeClusterDimension;
+  attr2[0].val.clusterDim.x = kCluster;
+  attr2[0].val.clusterDim.y = 1;
+  attr2[0].val.clusterDim.z = 1;
+  attr2[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr2[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr2;
+  cfg.numAttrs = 2;
+  return cudaLaunchKernelEx(&cfg, attn_tc_kernel<D>, tk, tv, a);
 }
 
 }  // namespace
 
-int attn_partitions(int capacity) { return (capacity + kPart - 1) / kPart; }
+int attn_q_tiles(int rows_per_request, int group) {
+  return (rows_per_request * group + kQT - 1) / kQT;
+}
+int attn_chunks(int capacity) { return (capacity + kChunk - 1) / kChunk; }
+size_t attn_qimg_bytes(int head_dim) { return (size_t)256 * head_dim; }
 
 cudaError_t launch_attention_split(const RowMap& m, const Model& md, KvState& kv, int layer,
                                    cudaStream_t st) {
   const as2d_config& c = md.cfg;
   AttnArgs a;
   a.rm = m;
-  a.q = kv.q;
   a.len = kv.d_len;
-  a.kc = kv.k_cache;
-  a.vc = kv.v_cache;
   a.layer = layer;
   a.batch = kv.batch;
   a.cap = kv.capacity;
   a.nq = c.n_q_heads;
   a.nkv = c.n_kv_heads;
   a.qscale = 1.4426950408889634f / sqrtf((float)c.head_dim);
-  a.ws_o = kv.attn_o;
-  a.ws_ml = kv.attn_ml;
-  a.parts_max = kv.attn_parts;
-  a.qmax = kv.attn_qmax;
-  a.ao = kv.ao;
-  a.lo_row = kv.rows_alloc;
-  int64_t max_len = 0;
-  a.part_start[0] = 0;
-  for (int b = 0; b < kv.batch; ++b) {
-    const int64_t e = kv.len_upper[b] + (m.start[b + 1] - m.start[b]);
-    max_len = e > max_len ? e : max_len;
-    a.part_start[b + 1] = a.part_start[b] + (int)((e + kPart - 1) / kPart);
-  }
-  const int parts = (int)((max_len + kPart - 1) / kPart);
-  const int items = a.part_start[kv.batch];
-  dim3 g1(items, c.n_kv_heads);
-  dim3 g2(m.rows, c.n_q_heads);
   a.qkv_part = kv.qkv_part;
   a.qkv_rinv = kv.qkv_rinv;
   a.rope = kv.rope;
   a.qkv_split = kv.qkv_split;
   a.qkv_ld = kv.rows_alloc;
-  const dim3 gf(m.rows, c.n_q_heads + 2 * c.n_kv_heads);
-  // merge groups for the call's longest row (each row uses min(4, its own
-  // partitions / 32 rounded up) of them)
-  int mg = (parts + 31) / 32;
-  mg = mg < 1 ? 1 : (mg > kMergeGroups ? kMergeGroups : mg);
-  // Eight warps stage a partition fastest; when there are more items than
-  // SMs, one warp per 16 query rows of the largest request (at least four,
-  // for the staging copies) lets two CTAs share an SM, so long prefixes need
-  // half the waves.  Which warp takes a row tile does not change its
-  // arithmetic.
-  int warps = 8;
-  if ((long long)items * c.n_kv_heads > md.sm_count) {
-    int qn_max = 0;
-    for (int b = 0; b < kv.batch; ++b) {
-      const int qn = (m.start[b + 1] - m.start[b]) * (c.n_q_heads / c.n_kv_heads);
-      qn_max = qn > qn_max ? qn : qn_max;
-    }
-    warps = (qn_max + 15) / 16;
-    warps = warps < 4 ? 4 : (warps > 8 ? 8 : warps);
+  a.kc = kv.k_cache;
+  a.vc = kv.v_cache;
+  a.qimg = kv.qimg;
+  a.qt_max = kv.attn_qt;
+  a.ws_o = kv.attn_o;
+  a.ws_ml = kv.attn_ml;
+  a.chunks_max = kv.attn_chunks;
+  a.cnt = kv.attn_cnt;
+  a.ao = kv.ao;
+  a.lo_row = kv.rows_alloc;
+  a.err = kv.d_err;
+  a.timeout_ns = 2000000000ull;
+  const int G = c.n_q_heads / c.n_kv_heads;
+  a.cl_start[0] = 0;
+  for (int b = 0; b < kv.batch; ++b) {
+    const int rows = m.start[b + 1] - m.start[b];
+    const int64_t keys = kv.len_upper[b] + rows;
+    int nch = (int)((keys + kChunk - 1) / kChunk);
+    if (nch > kv.attn_chunks) nch = kv.attn_chunks;
+    a.n_ch[b] = nch;
+    a.cl_start[b + 1] = a.cl_start[b] + attn_q_tiles(rows, G) * nch;
   }
-  const dim3 tpart(32 * warps);
+  const int clusters = a.cl_start[kv.batch];
+  const dim3 gf(m.rows, c.n_q_heads + 2 * c.n_kv_heads);
   cudaError_t e;
-  kv.launches += 3;
+  kv.launches += 2;
   if (c.head_dim == 128) {
     e = launch_pdl(qkv_finish_kernel<128>, gf, dim3(64), 0, st, a);
-    if (e == cudaSuccess) e = launch_pdl(attn_part_kernel<128>, g1, tpart, 0, st, a);
-    if (e == cudaSuccess) e = launch_pdl(attn_merge_kernel<128>, g2, dim3(128 * mg), 0, st, a);
+    if (e == cudaSuccess) e = launch_attn<128>(kv.tm_kc, kv.tm_vc, a, clusters, st);
   } else {
     e = launch_pdl(qkv_finish_kernel<64>, gf, dim3(32), 0, st, a);
-    if (e == cudaSuccess) e = launch_pdl(attn_part_kernel<64>, g1, tpart, 0, st, a);
-    if (e == cudaSuccess) e = launch_pdl(attn_merge_kernel<64>, g2, dim3(64 * mg), 0, st, a);
+    if (e == cudaSuccess) e = launch_attn<64>(kv.tm_kc, kv.tm_vc, a, clusters, st);
   }
   return e;
 }
