@@ -207,6 +207,18 @@ as2d_status as2d_kv_device_state(as2d_kv* kv, const int32_t** len,
    AS2D_OK. */
 as2d_status as2d_kv_check(as2d_kv* kv, void* stream);
 
+/* Time limit, in nanoseconds, of the waits inside the kernels of this state's
+   calls for a bulk copy, a tensor-core product or an accumulator (default
+   2 s; this file's failure detection, not a paper mechanism).  A wait that
+   runs out records AS2D_DEVERR_TIMEOUT, reported by as2d_kv_check, and its
+   block of threads abandons that call's work: the call's outputs are then
+   undefined, and the state should be restored with as2d_kv_rollback.  The
+   waits by which a block drains its own outstanding copies and products
+   before it ends keep the 2 s limit, so none is outstanding when it exits.
+   A limit of 0 makes every wait that is not already satisfied give up at
+   once, which exercises the failure path.  Takes effect for later calls. */
+as2d_status as2d_kv_set_wait_limit(as2d_kv* kv, uint64_t ns);
+
 /* One greedy decode step (k = 0) of a single request that allocates no
    memory.  The paper has no counterpart: this is for callers that must not
    allocate device memory when they decode -- for example a process whose

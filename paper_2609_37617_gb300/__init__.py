@@ -39,8 +39,8 @@ EXPORTED = ("as2d_model_load", "as2d_kv_init_prefilled", "as2d_verify_block",
             "as2d_decode_step", "as2d_kv_rollback", "as2d_kv_read_state",
             "as2d_kv_device_state", "as2d_kv_check", "as2d_kv_free",
             "as2d_model_free", "as2d_last_error", "as2d_kv_profile",
-            "as2d_kv_profile_read", "as2d_decode_step_static", "as2d_cbuf_create",
-            "as2d_cbuf_publish", "as2d_cbuf_candidates", "as2d_cbuf_after_call",
+            "as2d_kv_profile_read", "as2d_decode_step_static", "as2d_kv_set_wait_limit",
+            "as2d_cbuf_create", "as2d_cbuf_publish", "as2d_cbuf_candidates", "as2d_cbuf_after_call",
             "as2d_cbuf_state", "as2d_cbuf_source_of", "as2d_cbuf_free", "as2d_cbuf_held",
             "as2d_verify_from_buffers", "as2d_interval_accounting", "as2d_session_run",
             "as2d_budget_select", "as2d_prefill", "as2d_model_set_sm_budget",
@@ -123,6 +123,8 @@ _lib.as2d_kv_profile_read.argtypes = [_P, ctypes.POINTER(ctypes.c_int32),
                                       ctypes.POINTER(ctypes.c_int64)]
 _lib.as2d_kv_profile_read.restype = _S
 _lib.as2d_decode_step_static.argtypes = [_P, _P, _P, ctypes.c_int32, _P, _P, _P, _P, _P, _P]
+_lib.as2d_kv_set_wait_limit.argtypes = [_P, ctypes.c_uint64]
+_lib.as2d_kv_set_wait_limit.restype = _S
 _lib.as2d_decode_step_static.restype = _S
 _lib.as2d_cbuf_create.argtypes = [_S, ctypes.POINTER(ctypes.c_void_p)]
 _lib.as2d_cbuf_publish.argtypes = [_P, _P, _S, ctypes.POINTER(as2d_source_record)]
@@ -592,6 +594,9 @@ class State:
         st, n, ms, alln = as2d_kv_profile_read(self.handle)
         _check(st, "as2d_kv_profile_read")
         return n, ms, alln
+
+    def set_wait_limit(self, ns):
+        _check(_lib.as2d_kv_set_wait_limit(self.handle, int(ns)), "as2d_kv_set_wait_limit")
 
     def check(self, stream=0):
         _check(as2d_kv_check(self.handle, stream), "as2d_kv_check")

@@ -482,7 +482,7 @@ cudaError_t tc_project(int epi, const Model& m, KvState& s, const RowMap& rm, co
   p.ws = s.ws;
   p.counters = s.counters;
   p.err = s.d_err;
-  p.timeout_ns = 2000000000ull;
+  p.timeout_ns = s.wait_ns;
   p.rm = rm;
   for (int row0 = 0; row0 < rm.rows; row0 += 256) {
     p.row0 = row0;
@@ -611,6 +611,7 @@ extern "C" as2d_status as2d_prefill(as2d_kv* kh, const int32_t* tokens, int32_t 
   }
   KvState& w = *s.pf;
   w.len_upper = s.len_upper;
+  w.wait_ns = s.wait_ns;
   // passes of at most kPrefillRows tokens: the pass's first token stands in
   // for the pending root, the rest are kept as accepted candidates, and the
   // greedy token after the pass's last row becomes the root
@@ -710,6 +711,13 @@ extern "C" as2d_status as2d_kv_check(as2d_kv* kh, void* stream) {
     if (err & kErrCapacity) msg += " a device-side length left no room for the call's rows;";
     return fail(AS2D_ERR_DEVICE, msg);
   }
+  return AS2D_OK;
+}
+
+extern "C" as2d_status as2d_kv_set_wait_limit(as2d_kv* kh, uint64_t ns) {
+  g_err.clear();
+  if (!kh) return fail(AS2D_ERR_INVALID_ARG, "kv is NULL");
+  kh->s.wait_ns = ns;
   return AS2D_OK;
 }
 

@@ -190,6 +190,8 @@ struct KvState {
   CUtensorMap tm_xn[kNbCount], tm_ao[kNbCount], tm_u[kNbCount];
   // TMA descriptors of the caches: [n_layers * batch * n_kv][capacity][d]
   CUtensorMap tm_kc, tm_vc;
+  // limit of the kernels' pipeline waits (as2d_kv_set_wait_limit)
+  unsigned long long wait_ns = 2000000000ull;
   // measurement support
   int prof_class = -1;
   std::vector<cudaEvent_t> prof_events;  // pairs

@@ -436,7 +436,7 @@ __global__ void __launch_bounds__(192, 1)
       }
       // every copy this CTA issued has landed before the CTA may exit
       for (int j = (it > S ? it - S : 0); j < it; ++j)
-        ptx::mbar_wait(&full[j % S], (uint32_t)(j / S) & 1u, p.timeout_ns);
+        ptx::mbar_wait(&full[j % S], (uint32_t)(j / S) & 1u, ptx::kDrainNs);
     }
     __syncwarp();  // lanes 1..31 wait for lane 0: the warp reaches the barrier converged
   } else if (warp == 1) {
@@ -491,7 +491,7 @@ __global__ void __launch_bounds__(192, 1)
       }
       // every MMA this thread issued has completed before TMEM is freed
       ptx::mma_commit(drain);
-      ptx::mbar_wait(drain, 0, p.timeout_ns);
+      ptx::mbar_wait(drain, 0, ptx::kDrainNs);
     }
     __syncwarp();
   } else {

@@ -308,8 +308,8 @@ __global__ void __launch_bounds__(128, 2)
       if (tid == 0) {
         atomicOr(a.err, kErrTimeout);
         // the copies may still be in flight: wait for them before the CTA ends
-        ptx::mbar_wait(&bars[0], 0, a.timeout_ns);
-        ptx::mbar_wait(&bars[1], 0, a.timeout_ns);
+        ptx::mbar_wait(&bars[0], 0, ptx::kDrainNs);
+        ptx::mbar_wait(&bars[1], 0, ptx::kDrainNs);
       }
       __syncthreads();
     }
@@ -407,8 +407,8 @@ __global__ void __launch_bounds__(128, 2)
       if (tid == 0) {
         atomicOr(a.err, kErrTimeout);
         // no MMA may still run when TMEM is freed
-        ptx::mbar_wait(&bars[2], 0, a.timeout_ns);
-        if (ok1) ptx::mbar_wait(&bars[3], 0, a.timeout_ns);
+        ptx::mbar_wait(&bars[2], 0, ptx::kDrainNs);
+        if (ok1) ptx::mbar_wait(&bars[3], 0, ptx::kDrainNs);
       }
       m = -INFINITY;  // nothing of this tile is passed on
     }
@@ -621,7 +621,7 @@ cudaError_t launch_attention_split(const RowMap& m, const Model& md, KvState& kv
   a.ao = kv.ao;
   a.lo_row = kv.rows_alloc;
   a.err = kv.d_err;
-  a.timeout_ns = 2000000000ull;
+  a.timeout_ns = kv.wait_ns;
   const int G = c.n_q_heads / c.n_kv_heads;
   a.cl_start[0] = 0;
   for (int b = 0; b < kv.batch; ++b) {

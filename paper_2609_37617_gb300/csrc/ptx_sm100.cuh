@@ -54,15 +54,21 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 }
 
 // Wait for the phase with the given parity to complete, giving up after
-// `limit_ns` of wall time.  Returns false on timeout.
+// `limit_ns` of wall time (limit 0: at once, if it has not completed).
+// Returns false on timeout.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
-  for (uint32_t i = 1;; ++i) {
+  for (uint32_t i = 0;; ++i) {
     if (mbar_try_wait(bar, parity)) return true;
-    if ((i & 255u) == 0 && globaltimer_ns() - t0 > limit_ns) return false;
+    if ((i & 255u) == 0 && globaltimer_ns() - t0 >= limit_ns) return false;
   }
 }
+
+// Limit of the waits by which a CTA drains its own outstanding bulk copies
+// and tensor-core products before it exits: never shortened, so that no copy
+// or product is still outstanding when a CTA ends.
+constexpr uint64_t kDrainNs = 2000000000ull;
 
 // ---- TMA ------------------------------------------------------------------------
 

@@ -316,6 +316,37 @@ def test_max_batch_max_k_and_capacity_edge(pair):
     st.close()
 
 
+def test_bounded_wait_expiry_is_reported_and_recovers(pair):
+    """The kernels' bounded waits running out (failure detection, exercised
+    without a GPU fault): with a wait limit of 0 every wait that is not
+    already satisfied gives up at once, the call's blocks abandon their work
+    after draining their own copies and products, and as2d_kv_check reports
+    the timeout.  With the limit restored and the state rolled back, the next
+    call matches the oracle again."""
+    import torch
+    import paper_2609_37617_gb300 as lib
+    cfg = pair.cfg
+    root, oc, cont, cand = _workload_block(pair)
+    ores = pair.oracle.verify_block(oc, L0, root, cand)
+    st = pair.state([L0], CAP, [root])
+    st.set_wait_limit(0)
+    for _ in range(3):
+        run_gpu_block(st, cfg, [cand])
+        st.rollback([L0], [root])
+    torch.cuda.synchronize()
+    with pytest.raises(lib.AS2DError) as e:
+        st.check()
+    assert e.value.status == lib.AS2D_ERR_DEVICE
+    assert "timed out" in str(e.value)
+    st.check()                                # the flag was cleared
+    st.set_wait_limit(2_000_000_000)
+    st.rollback([L0], [root])
+    n, corr, greedy, logits = run_gpu_block(st, cfg, [cand])
+    compare_block(ores, logits[:5], greedy[:5], n[0], corr[0], 4)
+    st.check()
+    st.close()
+
+
 def test_zz_exact_checks_ran():
     """The module's bit-exact half ran: greedy rows and at least one full
     (n_accepted, correction) comparison (the sharp-model blocks above)."""
