@@ -311,7 +311,7 @@ as2d_status alloc_work(KvState& s, const Model& m, int batch, int capacity,
             encode_cache_map(&s.tm_vc, s.v_cache, m.cfg.head_dim, capacity,
                              (int64_t)m.cfg.n_layers * batch * m.cfg.n_kv_heads);
   for (int i = 0; i < kNbCount && ok; ++i) {
-    const int nb = 16 << i;
+    const int nb = kNbSet[i];
     if (nb > s.nb_max) break;
     ok = encode_2d(&s.tm_xn[i], s.xn, H, 2 * R, 64, nb) &&
          encode_2d(&s.tm_ao[i], s.ao, m.q_dim, 2 * R, 64, nb) &&

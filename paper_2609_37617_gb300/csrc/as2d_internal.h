@@ -136,12 +136,20 @@ struct Model {
   std::vector<const float*> attn_norm, mlp_norm;  // fp32 gains [H]
 };
 
-constexpr int kNbCount = 5;  // token-row paddings 16, 32, 64, 128, 256
-inline int nb_index(int nb) { return nb == 16 ? 0 : nb == 32 ? 1 : nb == 64 ? 2 : nb == 128 ? 3 : 4; }
+// Token-row paddings of the tensor-core projections (the MMA's N): a call of
+// `rows` token rows runs at the smallest one that holds them (at most 256 per
+// launch).  A row's arithmetic does not depend on the padding.
+constexpr int kNbCount = 10;
+constexpr int kNbSet[kNbCount] = {16, 32, 48, 64, 96, 128, 160, 192, 224, 256};
+inline int nb_index(int nb) {
+  int i = 0;
+  while (i + 1 < kNbCount && kNbSet[i] != nb) ++i;
+  return i;
+}
 inline int nb_for_rows(int rows) {
-  int nb = 16;
-  while (nb < rows && nb < 256) nb <<= 1;
-  return nb;
+  int i = 0;
+  while (i + 1 < kNbCount && kNbSet[i] < rows) ++i;
+  return kNbSet[i];
 }
 
 struct KvState {

@@ -46,12 +46,17 @@
 
 namespace as2d {
 
+// Weight-ring depth for a token-row padding: as many 16 KB weight tiles in
+// flight as the stage size (weights + the hi and lo activation tiles) allows.
+constexpr int tc_ring_depth(int nb) {
+  return nb <= 32 ? AS2D_RING16 : nb <= 64 ? 5 : nb <= 96 ? 4 : nb <= 192 ? 3 : 2;
+}
+
 template <int NB, int RING = 0>
 struct TcShape {
-  // ring depth: about 100 KB of weight tiles in flight per SM (RING: a
-  // shallower ring, so that a CTA fits on an SM beside an attention CTA)
-  static constexpr int S = RING ? RING
-                                : NB == 16 ? AS2D_RING16 : NB == 32 ? 6 : NB == 64 ? 5 : NB == 128 ? 3 : 2;
+  // ring depth (RING: a shallower ring, so that a CTA fits on an SM beside
+  // an attention CTA)
+  static constexpr int S = RING ? RING : tc_ring_depth(NB);
   static constexpr uint32_t A_BYTES = 128 * 64 * 2;
   static constexpr uint32_t B_BYTES = NB * 64 * 2;   // one of the hi / lo operand tiles
   static constexpr uint32_t STAGE_B = 2 * B_BYTES;   // hi tile, then lo tile
@@ -61,14 +66,20 @@ struct TcShape {
   // [NB, 2 NB), and are added in the epilogue (hi + lo) -- the same
   // arithmetic for every NB, so results stay batch invariant.  NB <= 128: one
   // MMA of N = 2 NB covers the hi and lo rows (adjacent in shared memory) and
-  // reads the weight tile once; NB = 256: two MMAs of N = 256.  Accumulators
-  // are double-buffered while 2 x 2 NB columns fit in TMEM's 512.
+  // reads the weight tile once; wider paddings: two MMAs of N = NB.
+  // Accumulators are double-buffered while 2 x 2 NB columns fit in TMEM's 512.
   static constexpr bool ONE_MMA = NB <= 128;
   static constexpr int ACC_COLS = 2 * NB;
   static constexpr int NBUF = 2 * ACC_COLS <= 512 ? 2 : 1;
-  static constexpr uint32_t TMEM_COLS = (NBUF * ACC_COLS < 32) ? 32 : NBUF * ACC_COLS;
+  static constexpr uint32_t TMEM_COLS = NBUF * ACC_COLS <= 32    ? 32
+                                        : NBUF * ACC_COLS <= 64  ? 64
+                                        : NBUF * ACC_COLS <= 128 ? 128
+                                        : NBUF * ACC_COLS <= 256 ? 256
+                                                                 : 512;
   static constexpr uint32_t SMEM =
       1024 + S * (A_BYTES + STAGE_B) + 128 * SP * 4 + (3 * NB + 64) * 4 + (2 * S + 5) * 8 + 16;
+  static_assert(SMEM <= 232448, "shared memory of one CTA");
+  static_assert(NB % 16 == 0 && NB >= 16 && NB <= 256, "MMA N of M = 128");
 };
 
 __device__ __forceinline__ float tc_silu(float x) { return x / (1.0f + expf(-x)); }
@@ -660,8 +671,13 @@ cudaError_t tc_gemm_dispatch(int nb, const CUtensorMap& x, const TcParams& p, cu
   switch (nb) {
     case 16: return tc_gemm_launch<16, EPI>(x, p, st);
     case 32: return tc_gemm_launch<32, EPI>(x, p, st);
+    case 48: return tc_gemm_launch<48, EPI>(x, p, st);
     case 64: return tc_gemm_launch<64, EPI>(x, p, st);
+    case 96: return tc_gemm_launch<96, EPI>(x, p, st);
     case 128: return tc_gemm_launch<128, EPI>(x, p, st);
+    case 160: return tc_gemm_launch<160, EPI>(x, p, st);
+    case 192: return tc_gemm_launch<192, EPI>(x, p, st);
+    case 224: return tc_gemm_launch<224, EPI>(x, p, st);
     case 256: return tc_gemm_launch<256, EPI>(x, p, st);
     default: return cudaErrorInvalidValue;
   }
