@@ -513,13 +513,12 @@ __global__ void __launch_bounds__(128, 2)
   __syncthreads();
   int* cnt = a.cnt + item * kCluster + rank;
   if (tid == 0) {
-    __threadfence();  // the CTA's writes above, before its arrival
-    const int prev = atomicAdd(cnt, 1);
+    // the arrival releases the CTA's writes above (ordered before it by the
+    // barrier) and acquires the other chunks' partials for the last arriver
+    int prev;
+    asm volatile("atom.add.acq_rel.gpu.s32 %0, [%1], 1;" : "=r"(prev) : "l"(cnt) : "memory");
     const int last = prev == n_chunks - 1;
-    if (last) {
-      *cnt = 0;  // every chunk of these rows has arrived
-      __threadfence();
-    }
+    if (last) *cnt = 0;  // every chunk of these rows has arrived
     *s_flag = last;
   }
   __syncthreads();
