@@ -39,7 +39,7 @@ WORKLOAD = "7b"
 
 # dram__bytes_read.sum + dram__bytes_write.sum per launch from one ncu capture
 # of the kernel as it stands (profiles/); None once the kernel has changed.
-TRAFFIC = {"gate_up": 275262720}  # 271,890,688 read + 3,372,032 written
+TRAFFIC = {"gate_up": 272226816}  # 271,882,752 read + 344,064 written
 
 # Diagnostic legs that reuse the headline state (each rolls it back to L0 first).
 BUDGET_WIN, BUDGET_COMMIT, BUDGET_TRACES = 220, 180, 4
@@ -535,6 +535,11 @@ def run_ours(args, ws, rank, local):
         "clocks": clk,
         "e2e": e2e,
         "errors": errors or None,
+        "profiles": {"launch_list": "profiles/launches_7b_k8_verify.md",
+                     "kernel_classes": "profiles/kernels_7b2l_k8_L1564.md",
+                     "attention": "profiles/attention_7b2l_k8.md",
+                     "gate_up": "profiles/gemm_gateup_7b_k8.md",
+                     "ragged": "profiles/kernels_7b2l_ragged16.md"},
     }
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = guarded(errors, "cpu_baseline", cpu_baseline, args, cfg, L0, plans)
