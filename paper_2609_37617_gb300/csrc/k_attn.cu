@@ -163,16 +163,18 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
-// Values x[0..7] of columns e0..e0+7 (e0 % 8 == 0) of query q, as bf16 hi
-// parts into row 2q and lo parts (x - hi) into row 2q + 1 of an operand image.
+// Values x[0..7] (>= 0) of columns e0..e0+7 (e0 % 8 == 0) of query q, as bf16
+// hi parts into row 2q and lo parts into row 2q + 1 of an operand image: hi =
+// x with its low 16 bits cleared (exact in bf16), lo = bf16(x - hi), so that
+// hi + lo matches x to about 17 bits.
 __device__ __forceinline__ void put_hilo8(uint8_t* img, int q, int e0, const float* x) {
   uint32_t hw[4], lw[4];
 #pragma unroll
   for (int u = 0; u < 4; ++u) {
-    const __nv_bfloat162 hv = __floats2bfloat162_rn(x[2 * u], x[2 * u + 1]);
-    const float2 hf = __bfloat1622float2(hv);
-    const __nv_bfloat162 lv = __floats2bfloat162_rn(x[2 * u] - hf.x, x[2 * u + 1] - hf.y);
-    hw[u] = *reinterpret_cast<const uint32_t*>(&hv);
+    const uint32_t b0 = __float_as_uint(x[2 * u]), b1 = __float_as_uint(x[2 * u + 1]);
+    hw[u] = (b0 >> 16) | (b1 & 0xFFFF0000u);
+    const __nv_bfloat162 lv = __floats2bfloat162_rn(x[2 * u] - __uint_as_float(b0 & 0xFFFF0000u),
+                                                    x[2 * u + 1] - __uint_as_float(b1 & 0xFFFF0000u));
     lw[u] = *reinterpret_cast<const uint32_t*>(&lv);
   }
   *reinterpret_cast<uint4*>(img + img_off(2 * q, e0)) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
@@ -356,17 +358,36 @@ __global__ void __launch_bounds__(128, 2)
         }
       }
       const int kb = p0 + 64 * pt;
-      float mx = -INFINITY;
+      // keys at or below the row's limit are visible; a half-tile wholly
+      // below it needs no mask (masked keys are skipped, never given -inf)
+      const bool all_vis = kb + 63 <= lim;
+      float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+      if (all_vis) {
 #pragma unroll
-      for (int j = 0; j < 64; ++j)
-        if (kb + j <= lim) mx = fmaxf(mx, sv[j]);
-      m = fmaxf(mx, __shfl_xor_sync(0xFFFFFFFFu, mx, 1));
-      float ls = 0.f;
+        for (int j = 0; j < 64; ++j) mx4[j & 3] = fmaxf(mx4[j & 3], sv[j]);
+      } else {
 #pragma unroll
-      for (int j = 0; j < 64; ++j) {
-        sv[j] = (kb + j <= lim) ? ex2(sv[j] - m) : 0.f;
-        ls += sv[j];
+        for (int j = 0; j < 64; ++j)
+          if (kb + j <= lim) mx4[j & 3] = fmaxf(mx4[j & 3], sv[j]);
       }
+      const float mx = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3]));
+      m = fmaxf(mx, __shfl_xor_sync(0xFFFFFFFFu, mx, 1));
+      // sums in four interleaved parts, then ((0 + 1) + (2 + 3)): a fixed order
+      float ls4[4] = {0.f, 0.f, 0.f, 0.f};
+      if (all_vis) {
+#pragma unroll
+        for (int j = 0; j < 64; ++j) {
+          sv[j] = ex2(sv[j] - m);
+          ls4[j & 3] += sv[j];
+        }
+      } else {
+#pragma unroll
+        for (int j = 0; j < 64; ++j) {
+          sv[j] = (kb + j <= lim) ? ex2(sv[j] - m) : 0.f;
+          ls4[j & 3] += sv[j];
+        }
+      }
+      const float ls = (ls4[0] + ls4[1]) + (ls4[2] + ls4[3]);
       const float lo_ = __shfl_xor_sync(0xFFFFFFFFu, ls, 1);
       l = pt ? lo_ + ls : ls + lo_;  // keys 0..63, then 64..127
       // P as bf16 hi (row 2q) and lo (row 2q + 1) parts, K-major by key
