@@ -295,6 +295,9 @@ __device__ __forceinline__ void tc_reduce_tile(const TcParams& p, float* sC, flo
   using Sh = TcShape<NB>;
   constexpr int CH = Sh::CH, SP = Sh::SP;
   const int nchunks = (p.rows + CH - 1) / CH;
+  // slot 1 holds a CTA's last segment when it began in an earlier tile: only
+  // the first part can be one
+  const int sl0 = (int)(tc_start(c_first, p) / p.kb) != tile ? 1 : 0;
   for (int ch = 0; ch < nchunks; ++ch) {
     const int live = p.rows - ch * CH;
     float acc[CH];
@@ -307,8 +310,7 @@ __device__ __forceinline__ void tc_reduce_tile(const TcParams& p, float* sC, flo
       for (int pp = 0; pp < MAXP; ++pp) {
         if (part0 + pp < nparts) {
           const int cp = c_first + part0 + pp;
-          // slot 1 holds a CTA's last segment when it began in an earlier tile
-          const int sl = (cp == c_first && (int)(tc_start(cp, p) / p.kb) != tile) ? 1 : 0;
+          const int sl = (part0 + pp == 0) ? sl0 : 0;
           const float* src = p.ws + ((size_t)(cp * 2 + sl) * NB + ch * CH) * 128 + nl;
 #pragma unroll
           for (int q = 0; q < 4; ++q)
@@ -417,13 +419,14 @@ __global__ void __launch_bounds__(192, 1)
         ptx::mbar_arrive_expect_tx(&full[it], A_BYTES + STAGE_B);
         ptx::bulk_load(sA + it * A_BYTES, p.w + (size_t)u * (128 * 64), A_BYTES, &full[it], pol_w);
       }
+      // k-block of each unit, stepped (no division after the wait)
+      int kb = (int)(u0 - (u0 / p.kb) * (long long)p.kb);
       ptx::griddep_wait();
       for (int it = 0; it < npre; ++it) {
-        const long long u = u0 + it;
-        const int kb = (int)(u - (u / p.kb) * (long long)p.kb);
         ptx::tma_load_2d(sB + it * STAGE_B, &tmX, &full[it], kb * 64, p.row0, pol_x);
         ptx::tma_load_2d(sB + it * STAGE_B + B_BYTES, &tmX, &full[it], kb * 64,
                          p.lo_row + p.row0, pol_x);
+        kb = (kb + 1 == p.kb) ? 0 : kb + 1;
       }
       int it = npre;
       bool ok = true;
@@ -434,12 +437,12 @@ __global__ void __launch_bounds__(192, 1)
           ok = false;
           break;
         }
-        const int kb = (int)(u - (u / p.kb) * (long long)p.kb);
         ptx::mbar_arrive_expect_tx(&full[s], A_BYTES + STAGE_B);
         ptx::bulk_load(sA + s * A_BYTES, p.w + (size_t)u * (128 * 64), A_BYTES, &full[s], pol_w);
         ptx::tma_load_2d(sB + s * STAGE_B, &tmX, &full[s], kb * 64, p.row0, pol_x);
         ptx::tma_load_2d(sB + s * STAGE_B + B_BYTES, &tmX, &full[s], kb * 64, p.lo_row + p.row0,
                          pol_x);
+        kb = (kb + 1 == p.kb) ? 0 : kb + 1;
       }
       if (!ok) {
         atomicOr(p.err, kErrTimeout);
@@ -613,6 +616,9 @@ __global__ void __launch_bounds__(128) tc_resid_finish_kernel(const __grid_const
   const int tile = blockIdx.x, m = blockIdx.y, n = threadIdx.x;
   const long long tstart = (long long)tile * p.kb, tend = tstart + p.kb;
   const int c_first = tc_owner(tstart, p), c_last = tc_owner(tend - 1, p);
+  // slot 1 holds a CTA's last segment when it began in an earlier tile: only
+  // the first part can be one
+  const int sl0 = (int)(tc_start(c_first, p) / p.kb) != tile ? 1 : 0;
   ptx::griddep_wait();
   ptx::griddep_launch_dependents();
   if (c_last == c_first) return;  // a whole tile, finished by its GEMM CTA
@@ -620,6 +626,7 @@ __global__ void __launch_bounds__(128) tc_resid_finish_kernel(const __grid_const
   const int col = tile * 128 + n;
   const size_t at = (size_t)(p.row0 + m) * p.N + col;
   const float h0 = p.h[at], gn = p.g_next[col];
+  const float* src = p.ws + (size_t)m * 128 + n;
   float acc = 0.f;
   for (int part0 = 0; part0 < nparts; part0 += 8) {
     float v[8];
@@ -628,8 +635,8 @@ __global__ void __launch_bounds__(128) tc_resid_finish_kernel(const __grid_const
       v[pp] = 0.f;
       if (part0 + pp < nparts) {
         const int cp = c_first + part0 + pp;
-        const int sl = (cp == c_first && (int)(tc_start(cp, p) / p.kb) != tile) ? 1 : 0;
-        v[pp] = __ldcg(p.ws + ((size_t)(cp * 2 + sl) * NB + m) * 128 + n);
+        const int sl = (part0 + pp == 0) ? sl0 : 0;
+        v[pp] = __ldcg(src + (size_t)(cp * 2 + sl) * NB * 128);
       }
     }
 #pragma unroll
