@@ -458,15 +458,19 @@ cudaError_t tc_project(int epi, const Model& m, KvState& s, const RowMap& rm, co
   // row's sums are added in the same order whatever the number of rows):
   //   QKV (TC_PART): K split evenly over qkv_split CTAs per tile, sums
   //     finished by qkv_finish_kernel;
-  //   at least as many tiles as SMs (gate/up): whole tiles per CTA, as
-  //     evenly as they go, each finished by its own CTA;
-  //   otherwise stream-K over one CTA per SM; residual projections leave
-  //     their split tiles to tc_resid_finish_kernel, the LM head finishes
-  //     them in the GEMM (last CTA of a tile).
+  //   at least 90% as many tiles as SMs (gate/up): whole tiles per CTA,
+  //     as evenly as they go, each finished by its own CTA;
+  //   otherwise stream-K over one CTA per SM, with at least four units per
+  //     CTA for the residual projections (a small projection spread over
+  //     every SM cuts each tile into many parts, and its CTAs on SMs still
+  //     held by the attention start late); residual projections leave their
+  //     split tiles to tc_resid_finish_kernel, the LM head finishes them in
+  //     the GEMM (last CTA of a tile).
   p.grid = (int)(p.units < m.sm_count ? p.units : m.sm_count);
+  if (epi == TC_RESID && p.units / 4 < p.grid) p.grid = p.units >= 4 ? (int)(p.units / 4) : 1;
   p.split = 0;
   p.defer = epi == TC_RESID ? 1 : 0;
-  if (epi == TC_SWIGLU && p.n_tiles >= m.sm_count) {
+  if (epi == TC_SWIGLU && p.n_tiles * 10 >= m.sm_count * 9) {
     const int per = (p.n_tiles + m.sm_count - 1) / m.sm_count;
     p.split = 1;
     p.grid = (p.n_tiles + per - 1) / per;

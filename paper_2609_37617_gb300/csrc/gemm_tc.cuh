@@ -628,10 +628,10 @@ __global__ void __launch_bounds__(128) tc_resid_finish_kernel(const __grid_const
   const float h0 = p.h[at], gn = p.g_next[col];
   const float* src = p.ws + (size_t)m * 128 + n;
   float acc = 0.f;
-  for (int part0 = 0; part0 < nparts; part0 += 8) {
-    float v[8];
+  for (int part0 = 0; part0 < nparts; part0 += 16) {
+    float v[16];
 #pragma unroll
-    for (int pp = 0; pp < 8; ++pp) {
+    for (int pp = 0; pp < 16; ++pp) {
       v[pp] = 0.f;
       if (part0 + pp < nparts) {
         const int cp = c_first + part0 + pp;
@@ -640,7 +640,7 @@ __global__ void __launch_bounds__(128) tc_resid_finish_kernel(const __grid_const
       }
     }
 #pragma unroll
-    for (int pp = 0; pp < 8; ++pp)
+    for (int pp = 0; pp < 16; ++pp)
       if (part0 + pp < nparts) acc += v[pp];
   }
   const float hn = h0 + acc;

@@ -120,12 +120,15 @@ __global__ void __launch_bounds__(D / 2) qkv_finish_kernel(AttnArgs a) {
   constexpr int H2 = D / 2;
   const int gm = blockIdx.x, head = blockIdx.y, e = threadIdx.x;
   const int b = row_request(a.rm, gm), i = gm - a.rm.start[b];
-  if (!rows_fit(a.len[b], a.rm.start[b + 1] - a.rm.start[b], a.cap)) return;  // flagged
-  const int pos = a.len[b] + i;
-  float y0, y1;
+  // every load is issued before any is used: one memory round trip
+  const int len_b = a.len[b];
   const float x = qkv_value(a, head * D + e, gm), xp = qkv_value(a, head * D + e + H2, gm);
-  if (head < a.nq + a.nkv) {
-    const float2 cs = a.rope[(size_t)gm * H2 + e];
+  const bool rotate = head < a.nq + a.nkv;
+  const float2 cs = rotate ? a.rope[(size_t)gm * H2 + e] : make_float2(1.f, 0.f);
+  if (!rows_fit(len_b, a.rm.start[b + 1] - a.rm.start[b], a.cap)) return;  // flagged
+  const int pos = len_b + i;
+  float y0, y1;
+  if (rotate) {
     y0 = fmaf(x, cs.x, -(xp * cs.y));
     y1 = fmaf(xp, cs.x, x * cs.y);
   } else {
@@ -544,16 +547,15 @@ __global__ void __launch_bounds__(128, 2)
   }
   __syncthreads();
   if (!*s_flag) return;
-  float cm = -INFINITY;
-  for (int cc = 0; cc < n_chunks; ++cc)
-    cm = fmaxf(cm, __ldcg(a.ws_ml + (item * a.chunks_max + cc) * kQT + fr).x);
   float cl_ = 0.f, co[DT];
 #pragma unroll
   for (int e = 0; e < DT; ++e) co[e] = 0.f;
-  for (int c0 = 0; c0 < n_chunks; c0 += 8) {
-    // eight chunks' values in flight at a time
-    float4 v[8][DT / 4];
-    float2 ml[8];
+  // eight chunks' values in flight at a time; the first eight are requested
+  // together with every chunk's maximum, so that up to eight chunks take one
+  // memory round trip
+  float4 v[8][DT / 4];
+  float2 ml[8];
+  auto load8 = [&](int c0) {
 #pragma unroll
     for (int u8 = 0; u8 < 8; ++u8)
       if (c0 + u8 < n_chunks) {
@@ -563,6 +565,16 @@ __global__ void __launch_bounds__(128, 2)
 #pragma unroll
         for (int u = 0; u < DT / 4; ++u) v[u8][u] = __ldcg(src + u);
       }
+  };
+  load8(0);
+  float cm = -INFINITY;
+  for (int cc = 8; cc < n_chunks; ++cc)
+    cm = fmaxf(cm, __ldcg(a.ws_ml + (item * a.chunks_max + cc) * kQT + fr).x);
+#pragma unroll
+  for (int u8 = 0; u8 < 8; ++u8)
+    if (u8 < n_chunks) cm = fmaxf(cm, ml[u8].x);
+  for (int c0 = 0; c0 < n_chunks; c0 += 8) {
+    if (c0 > 0) load8(c0);
 #pragma unroll
     for (int u8 = 0; u8 < 8; ++u8)
       if (c0 + u8 < n_chunks) {
