@@ -228,9 +228,10 @@ __global__ void __launch_bounds__(128, 2)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  uint8_t* R0 = sm;            // Q image -> P image -> the partials received from the cluster
-  uint8_t* R1 = sm + 32768;    // K tile
+  uint8_t* R0 = sm;            // Q image -> P image
+  uint8_t* R1 = sm + 32768;    // K tile -> the partials received from the cluster
   uint8_t* R2 = sm + 65536;    // V tile
+  float* recv = reinterpret_cast<float*>(R1);  // [8 tiles][8 rows][D] received
   float2* s_rml = reinterpret_cast<float2*>(sm + 98304);  // [8 tiles][8 rows] received (max, sum)
   float* s_x = reinterpret_cast<float*>(s_rml + 64);      // [8] scratch
   uint64_t* bars = reinterpret_cast<uint64_t*>(s_x + 8);  // q, kv, mma1, mma2
@@ -254,6 +255,7 @@ __global__ void __launch_bounds__(128, 2)
   const int n_chunks = (n_tiles + kCluster - 1) / kCluster;
   const bool active = t < n_tiles;      // this CTA's tile holds keys
   const bool cl_active = c < n_chunks;  // uniform over the cluster
+  if (!cl_active) return;               // the whole cluster holds no keys of this request
   const int z = (a.layer * a.batch + b) * a.nkv + g;
   const uint8_t* qsrc = a.qimg + ((size_t)(b * a.nkv + g) * a.qt_max + qt) * (size_t)Q_BYTES;
 
@@ -344,6 +346,12 @@ __global__ void __launch_bounds__(128, 2)
       ptx::fence_proxy_async_smem();
     }
     const bool ok1 = ptx::group_all(ptx::mbar_wait(&bars[2], 0, a.timeout_ns), 1, 128);
+    // the tile's keys are consumed (after a timeout: once the product has
+    // drained), so its K image may receive the cluster's partials; the
+    // others wait for this arrival only when they push, after their own
+    // second product
+    if (!ok1 && tid == 0) ptx::mbar_wait(&bars[2], 0, ptx::kDrainNs);
+    ptx::cluster_arrive_release();
     ptx::tc_fence_after();
     bool ok2 = ok1;
     if (ok1) {
@@ -436,24 +444,25 @@ __global__ void __launch_bounds__(128, 2)
       }
       m = -INFINITY;  // nothing of this tile is passed on
     }
+  } else {
+    ptx::cluster_arrive_release();  // no keys of this CTA's tile are read
   }
   ptx::tc_fence_before();
   __syncthreads();
   if (warp == 0) ptx::tmem_dealloc(tmem, 256);
-  if (!cl_active) return;  // the whole cluster holds no keys of this request
 
   // ---- the cluster's tile partials, pushed to the CTA that folds them ----
   // CTA r folds query rows 8r..8r+7; it receives, from every CTA i of the
-  // cluster, rows (max, sum) into s_rml[i][row] and O into its R0 as
-  // [i][row][d] (every CTA's P image is consumed once all pass this barrier)
-  ptx::cluster_sync();
+  // cluster, rows (max, sum) into s_rml[i][row] and O into recv[i][row][d],
+  // over its K image (every CTA's K image is consumed once all have arrived)
+  ptx::cluster_wait();
   if (active) {
     const uint32_t dst_rank = (uint32_t)(q >> 3), row = (uint32_t)(q & 7);
     if (pt == 0)
       dsmem_st_f2(ptx::dsmem_map(ptx::smem_u32(s_rml + rank * 8 + row), dst_rank), make_float2(m, l));
     if (m != -INFINITY) {
-      const uint32_t dst = ptx::dsmem_map(
-          ptx::smem_u32(reinterpret_cast<float*>(R0) + (rank * 8 + row) * D + pt * DH), dst_rank);
+      const uint32_t dst =
+          ptx::dsmem_map(ptx::smem_u32(recv + (rank * 8 + row) * D + pt * DH), dst_rank);
 #pragma unroll
       for (int u = 0; u < DH / 4; ++u)
         dsmem_st_f4(dst + 16u * u, make_float4(o[4 * u], o[4 * u + 1], o[4 * u + 2], o[4 * u + 3]));
@@ -479,8 +488,7 @@ __global__ void __launch_bounds__(128, 2)
     const float w = part_weight(pml[i].x, fm);
     if (w != 0.f) {
       fl += pml[i].y * w;
-      const float4* src = reinterpret_cast<const float4*>(reinterpret_cast<float*>(R0) +
-                                                          (i * 8 + fj) * D + fd);
+      const float4* src = reinterpret_cast<const float4*>(recv + (i * 8 + fj) * D + fd);
 #pragma unroll
       for (int u = 0; u < DT / 4; ++u) {
         const float4 v = src[u];

@@ -279,6 +279,17 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
 
 // Every thread of every CTA of the cluster arrives, then waits for all:
 // shared-memory writes before it are visible to the cluster after it.
+// The two halves of a cluster barrier, for a split arrival: arrive
+// (release: this thread's earlier accesses, and those its CTA ordered before
+// it, happen before the others' accesses after their wait) and wait.
+// Every thread of every CTA of the cluster takes part.
+__device__ __forceinline__ void cluster_arrive_release() {
+  asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait() {
+  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
 __device__ __forceinline__ void cluster_sync() {
   asm volatile(
       "barrier.cluster.arrive.release.aligned;\n\t"
