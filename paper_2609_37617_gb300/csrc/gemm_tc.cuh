@@ -619,13 +619,16 @@ __global__ void __launch_bounds__(128) tc_resid_finish_kernel(const __grid_const
   // slot 1 holds a CTA's last segment when it began in an earlier tile: only
   // the first part can be one
   const int sl0 = (int)(tc_start(c_first, p) / p.kb) != tile ? 1 : 0;
+  const int col = tile * 128 + n;
+  // the next norm's gain is a weight, written by no kernel: its load (often
+  // from HBM, busy with the next projection's weight stream) overlaps the wait
+  const float gn = c_last != c_first ? __ldg(p.g_next + col) : 0.f;
   ptx::griddep_wait();
   ptx::griddep_launch_dependents();
   if (c_last == c_first) return;  // a whole tile, finished by its GEMM CTA
   const int nparts = c_last - c_first + 1;
-  const int col = tile * 128 + n;
   const size_t at = (size_t)(p.row0 + m) * p.N + col;
-  const float h0 = p.h[at], gn = p.g_next[col];
+  const float h0 = p.h[at];
   const float* src = p.ws + (size_t)m * 128 + n;
   float acc = 0.f;
   for (int part0 = 0; part0 < nparts; part0 += 16) {
