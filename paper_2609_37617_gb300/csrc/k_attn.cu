@@ -55,7 +55,18 @@ constexpr int kCluster = 8;   // CTAs per cluster
 constexpr int kChunk = kTile * kCluster;
 constexpr int kQT = 64;       // queries per query tile (hi and lo rows interleaved)
 constexpr uint32_t kRegion = 128 * 128;  // one 64-column region of 128 rows, bytes
-constexpr uint32_t kSmemAttn = 3 * 32768 + 64 * 8 + 8 * 4 + 4 * 8 + 16 + 1024;
+// Shared memory: the Q / P image, then the K and V tiles.  Wide (one wave of
+// clusters): K and V in separate images, both requested at the start.
+// Narrow (launches of several waves): V is loaded over K once the first
+// product has consumed it, so that three CTAs fit on an SM.
+template <bool NARROW>
+constexpr uint32_t attn_smem() {
+  return (NARROW ? 2 : 3) * 32768 + 64 * 8 + 8 * 4 + 5 * 8 + 16 + 1024;
+}
+static_assert(3 * (attn_smem<true>() + 1024) <= 228 * 1024, "three narrow CTAs per SM");
+// at most this many clusters of 8 run at once (cudaOccupancyMaxActiveClusters
+// of the wide kernel); a launch with more takes the narrow layout
+constexpr int kWideClusters = 15;
 
 struct AttnArgs {
   RowMap rm;
@@ -216,12 +227,13 @@ __device__ __forceinline__ float part_weight(float m, float M) {
   return m == -INFINITY ? 0.f : (m == M ? 1.f : ex2(m - M));
 }
 
-template <int D>
-__global__ void __launch_bounds__(128, 2)
+template <int D, bool NARROW>
+__global__ void __launch_bounds__(128, NARROW ? 3 : 2)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
                    const __grid_constant__ AttnArgs a) {
   constexpr int NR = D / 64;          // 64-column regions of a K / V tile
-  constexpr uint32_t KV_BYTES = 2u * NR * kRegion;
+  constexpr uint32_t K_BYTES = NR * kRegion;            // one K or V tile
+  constexpr uint32_t TMEM_COLS = NARROW ? 128 : 256;   // narrow: O over S
   constexpr uint32_t Q_BYTES = 2u * kQT * D * 2;
   constexpr int DH = D / 2;           // dims each thread of a hi/lo pair keeps
   constexpr int DT = D / 16;          // dims per thread in the folds (8 rows x 16 threads)
@@ -230,12 +242,12 @@ __global__ void __launch_bounds__(128, 2)
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   uint8_t* R0 = sm;            // Q image -> P image
   uint8_t* R1 = sm + 32768;    // K tile -> the partials received from the cluster
-  uint8_t* R2 = sm + 65536;    // V tile
+  uint8_t* R2 = NARROW ? R1 : sm + 65536;  // V tile (narrow: over K, after the first product)
   float* recv = reinterpret_cast<float*>(R1);  // [8 tiles][8 rows][D] received
-  float2* s_rml = reinterpret_cast<float2*>(sm + 98304);  // [8 tiles][8 rows] received (max, sum)
+  float2* s_rml = reinterpret_cast<float2*>(sm + (NARROW ? 2 : 3) * 32768);  // [8][8] (max, sum)
   float* s_x = reinterpret_cast<float*>(s_rml + 64);      // [8] scratch
-  uint64_t* bars = reinterpret_cast<uint64_t*>(s_x + 8);  // q, kv, mma1, mma2
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 4);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(s_x + 8);  // q, k (wide: and v), mma1, mma2, v
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 5);
   int* s_flag = reinterpret_cast<int*>(tslot + 1);
 
   const int tid = threadIdx.x, warp = tid >> 5;
@@ -260,10 +272,10 @@ __global__ void __launch_bounds__(128, 2)
   const uint8_t* qsrc = a.qimg + ((size_t)(b * a.nkv + g) * a.qt_max + qt) * (size_t)Q_BYTES;
 
   if (tid == 0) {
-    for (int i = 0; i < 4; ++i) ptx::mbar_init(&bars[i], 1);
+    for (int i = 0; i < 5; ++i) ptx::mbar_init(&bars[i], 1);
     ptx::fence_mbar_init();
   }
-  if (warp == 0) ptx::tmem_alloc(tslot, 256);
+  if (warp == 0) ptx::tmem_alloc(tslot, TMEM_COLS);
   ptx::tc_fence_before();
   __syncthreads();
   ptx::tc_fence_after();
@@ -275,12 +287,17 @@ __global__ void __launch_bounds__(128, 2)
   const bool early = active && p0 + kTile <= L;
   const uint64_t pol = ptx::policy_evict_first();
   auto load_kv = [&]() {
-    ptx::mbar_arrive_expect_tx(&bars[1], KV_BYTES);
+    ptx::mbar_arrive_expect_tx(&bars[1], NARROW ? K_BYTES : 2 * K_BYTES);
 #pragma unroll
     for (int h = 0; h < NR; ++h) {
       ptx::tma_load_3d(R1 + h * kRegion, &tmK, &bars[1], 64 * h, p0, z, pol);
-      ptx::tma_load_3d(R2 + h * kRegion, &tmV, &bars[1], 64 * h, p0, z, pol);
+      if (!NARROW) ptx::tma_load_3d(R2 + h * kRegion, &tmV, &bars[1], 64 * h, p0, z, pol);
     }
+  };
+  auto load_v = [&]() {  // narrow: into the K image, once the first product is done
+    ptx::mbar_arrive_expect_tx(&bars[4], K_BYTES);
+#pragma unroll
+    for (int h = 0; h < NR; ++h) ptx::tma_load_3d(R2 + h * kRegion, &tmV, &bars[4], 64 * h, p0, z, pol);
   };
   if (tid == 0 && early) {
     ptx::prefetch_tmap(&tmK);
@@ -321,6 +338,23 @@ __global__ void __launch_bounds__(128, 2)
       __syncthreads();
     }
   }
+  // values past the call's last key (stale entries, or NaN in a poisoned
+  // cache) would reach O through 0 * V: those rows of the V tile are zeroed
+  auto zero_v_tail = [&]() {
+    const int z0 = kend - p0;
+    if (z0 < kTile) {
+      for (int idx = tid; idx < (kTile - z0) * NR * 8; idx += 128) {
+        const int r = z0 + idx / (NR * 8), rest = idx - (idx / (NR * 8)) * (NR * 8);
+        *reinterpret_cast<uint4*>(R2 + (rest >> 3) * kRegion + r * 128 + (rest & 7) * 16) =
+            make_uint4(0, 0, 0, 0);
+      }
+      ptx::fence_proxy_async_smem();
+    }
+  };
+  // Every thread arrives once at the split cluster barrier, when its CTA no
+  // longer reads the image the cluster's partials are received into (the K
+  // image: wide after the first product, narrow after the second, V being
+  // loaded there).  The others wait for the arrival only when they push.
   if (active && ok) {
     if (tid == 0) {
       ptx::tc_fence_after();
@@ -333,27 +367,15 @@ __global__ void __launch_bounds__(128, 2)
       }
       ptx::mma_commit(&bars[2]);
     }
-    // values past the call's last key (stale entries, or NaN in a poisoned
-    // cache) would reach O through 0 * V: zero those rows of the V tile
-    // while the first product runs
-    const int z0 = kend - p0;
-    if (z0 < kTile) {
-      for (int idx = tid; idx < (kTile - z0) * NR * 8; idx += 128) {
-        const int r = z0 + idx / (NR * 8), rest = idx - (idx / (NR * 8)) * (NR * 8);
-        *reinterpret_cast<uint4*>(R2 + (rest >> 3) * kRegion + r * 128 + (rest & 7) * 16) =
-            make_uint4(0, 0, 0, 0);
-      }
-      ptx::fence_proxy_async_smem();
-    }
+    if (!NARROW) zero_v_tail();  // while the first product runs
     const bool ok1 = ptx::group_all(ptx::mbar_wait(&bars[2], 0, a.timeout_ns), 1, 128);
-    // the tile's keys are consumed (after a timeout: once the product has
-    // drained), so its K image may receive the cluster's partials; the
-    // others wait for this arrival only when they push, after their own
-    // second product
+    // (after a timeout: once the product has drained)
     if (!ok1 && tid == 0) ptx::mbar_wait(&bars[2], 0, ptx::kDrainNs);
-    ptx::cluster_arrive_release();
+    if (!NARROW || !ok1) ptx::cluster_arrive_release();
+    // narrow: the keys are consumed; V comes into their image during the softmax
+    if (NARROW && ok1 && tid == 0) load_v();
     ptx::tc_fence_after();
-    bool ok2 = ok1;
+    bool ok2 = ok1, vok = ok1;
     if (ok1) {
       // S = hi + lo of this thread's keys, masked; the tile's maximum and
       // P = 2^(S - m) with the partner lane
@@ -404,27 +426,41 @@ __global__ void __launch_bounds__(128, 2)
       // P as bf16 hi (row 2q) and lo (row 2q + 1) parts, K-major by key
 #pragma unroll
       for (int ch = 0; ch < 8; ++ch) put_hilo8(R0, q, 64 * pt + 8 * ch, sv + 8 * ch);
+      if (NARROW) {
+        vok = ptx::group_all(ptx::mbar_wait(&bars[4], 0, a.timeout_ns), 1, 128);
+        if (vok) zero_v_tail();
+      }
       ptx::fence_proxy_async_smem();
+      // (narrow: the second product writes O over S, read out above)
+      ptx::tc_fence_before();
       __syncthreads();
-      if (tid == 0) {
+      if (tid == 0 && vok) {
         ptx::tc_fence_after();
         constexpr uint32_t IDESC2 = ptx::idesc_bf16_f32(128, D, true);
 #pragma unroll
         for (int kk = 0; kk < kTile / 16; ++kk) {
           const uint64_t ad = ptx::sdesc_sw128(ptx::smem_u32(R0 + (kk >> 2) * kRegion)) + 2 * (kk & 3);
           const uint64_t bd = ptx::sdesc_sw128_mn(ptx::smem_u32(R2) + kk * 2048u, kRegion, 1024u);
-          ptx::mma_bf16(tmem + 128, ad, bd, IDESC2, kk > 0 ? 1u : 0u);
+          ptx::mma_bf16(tmem + (NARROW ? 0 : 128), ad, bd, IDESC2, kk > 0 ? 1u : 0u);
         }
         ptx::mma_commit(&bars[3]);
       }
-      ok2 = ptx::group_all(ptx::mbar_wait(&bars[3], 0, a.timeout_ns), 1, 128);
+      ok2 = vok && ptx::group_all(ptx::mbar_wait(&bars[3], 0, a.timeout_ns), 1, 128);
+      if (NARROW) {
+        // (after a timeout: once the copy and the product have drained)
+        if (!ok2 && tid == 0) {
+          ptx::mbar_wait(&bars[4], 0, ptx::kDrainNs);
+          if (vok) ptx::mbar_wait(&bars[3], 0, ptx::kDrainNs);
+        }
+        ptx::cluster_arrive_release();
+      }
       ptx::tc_fence_after();
       if (ok2) {
         // O = hi + lo of this thread's dims
 #pragma unroll
         for (int c0 = 0; c0 < D; c0 += 64) {
           float v[64];
-          tmem_ld64(tmem + lane_base + 128 + c0, v);
+          tmem_ld64(tmem + lane_base + (NARROW ? 0 : 128) + c0, v);
 #pragma unroll
           for (int j = 0; j < 64; ++j) {
             const int d = c0 + j;  // compile-time after unrolling
@@ -440,7 +476,7 @@ __global__ void __launch_bounds__(128, 2)
         atomicOr(a.err, kErrTimeout);
         // no MMA may still run when TMEM is freed
         ptx::mbar_wait(&bars[2], 0, ptx::kDrainNs);
-        if (ok1) ptx::mbar_wait(&bars[3], 0, ptx::kDrainNs);
+        if (vok) ptx::mbar_wait(&bars[3], 0, ptx::kDrainNs);
       }
       m = -INFINITY;  // nothing of this tile is passed on
     }
@@ -449,12 +485,12 @@ __global__ void __launch_bounds__(128, 2)
   }
   ptx::tc_fence_before();
   __syncthreads();
-  if (warp == 0) ptx::tmem_dealloc(tmem, 256);
+  if (warp == 0) ptx::tmem_dealloc(tmem, TMEM_COLS);
 
   // ---- the cluster's tile partials, pushed to the CTA that folds them ----
   // CTA r folds query rows 8r..8r+7; it receives, from every CTA i of the
   // cluster, rows (max, sum) into s_rml[i][row] and O into recv[i][row][d],
-  // over its K image (every CTA's K image is consumed once all have arrived)
+  // over its K image (every CTA's is consumed once all have arrived)
   ptx::cluster_wait();
   if (active) {
     const uint32_t dst_rank = (uint32_t)(q >> 3), row = (uint32_t)(q & 7);
@@ -602,16 +638,17 @@ __global__ void __launch_bounds__(128, 2)
   write_out(co, cl_);
 }
 
-template <int D>
+template <int D, bool NARROW>
 cudaError_t launch_attn(const CUtensorMap& tk, const CUtensorMap& tv, const AttnArgs& a,
                         int clusters, cudaStream_t st) {
+  constexpr uint32_t smem = attn_smem<NARROW>();
   static const cudaError_t attr = cudaFuncSetAttribute(
-      attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemAttn);
+      attn_tc_kernel<D, NARROW>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (attr != cudaSuccess) return attr;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(clusters * kCluster, a.nkv);
   cfg.blockDim = dim3(128);
-  cfg.dynamicSmemBytes = kSmemAttn;
+  cfg.dynamicSmemBytes = smem;
   cfg.stream = st;
   cudaLaunchAttribute attr2[2];
   attr2[0].id = cudaLaunchAttributeClusterDimension;
@@ -622,7 +659,7 @@ cudaError_t launch_attn(const CUtensorMap& tk, const CUtensorMap& tv, const Attn
   attr2[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr2;
   cfg.numAttrs = 2;
-  return cudaLaunchKernelEx(&cfg, attn_tc_kernel<D>, tk, tv, a);
+  return cudaLaunchKernelEx(&cfg, attn_tc_kernel<D, NARROW>, tk, tv, a);
 }
 
 }  // namespace
@@ -673,15 +710,22 @@ cudaError_t launch_attention_split(const RowMap& m, const Model& md, KvState& kv
     a.cl_start[b + 1] = a.cl_start[b] + attn_q_tiles(rows, G) * nch;
   }
   const int clusters = a.cl_start[kv.batch];
+  // the same arithmetic either way: the layout only decides how many CTAs an
+  // SM holds
+  const bool narrow = clusters * c.n_kv_heads > kWideClusters;
   const dim3 gf(m.rows, c.n_q_heads + 2 * c.n_kv_heads);
   cudaError_t e;
   kv.launches += 2;
   if (c.head_dim == 128) {
     e = launch_pdl(qkv_finish_kernel<128>, gf, dim3(64), 0, st, a);
-    if (e == cudaSuccess) e = launch_attn<128>(kv.tm_kc, kv.tm_vc, a, clusters, st);
+    if (e == cudaSuccess)
+      e = narrow ? launch_attn<128, true>(kv.tm_kc, kv.tm_vc, a, clusters, st)
+                 : launch_attn<128, false>(kv.tm_kc, kv.tm_vc, a, clusters, st);
   } else {
     e = launch_pdl(qkv_finish_kernel<64>, gf, dim3(32), 0, st, a);
-    if (e == cudaSuccess) e = launch_attn<64>(kv.tm_kc, kv.tm_vc, a, clusters, st);
+    if (e == cudaSuccess)
+      e = narrow ? launch_attn<64, true>(kv.tm_kc, kv.tm_vc, a, clusters, st)
+                 : launch_attn<64, false>(kv.tm_kc, kv.tm_vc, a, clusters, st);
   }
   return e;
 }
