@@ -59,11 +59,16 @@ constexpr uint32_t kRegion = 128 * 128;  // one 64-column region of 128 rows, by
 // clusters): K and V in separate images, both requested at the start.
 // Narrow (launches of several waves): V is loaded over K once the first
 // product has consumed it, so that three CTAs fit on an SM.
-template <bool NARROW>
+// Pair (wide only): clusters of 16 CTAs, two chunks, whose second chunk's
+// partial comes to the first chunk's CTAs through distributed shared memory
+// ([8 rows][d] floats and [8] (max, sum)) instead of through global memory.
+template <bool NARROW, bool PAIR>
 constexpr uint32_t attn_smem() {
-  return (NARROW ? 2 : 3) * 32768 + 64 * 8 + 8 * 4 + 5 * 8 + 16 + 1024;
+  return (NARROW ? 2 : 3) * 32768 + 64 * 8 + 8 * 4 + 5 * 8 + 16 +
+         (PAIR ? 16 + 8 * 128 * 4 + 8 * 8 : 0) + 1024;
 }
-static_assert(3 * (attn_smem<true>() + 1024) <= 228 * 1024, "three narrow CTAs per SM");
+static_assert(3 * (attn_smem<true, false>() + 1024) <= 228 * 1024, "three narrow CTAs per SM");
+static_assert(2 * (attn_smem<false, true>() + 1024) <= 228 * 1024, "two wide CTAs per SM");
 // at most this many clusters of 8 run at once (cudaOccupancyMaxActiveClusters
 // of the wide kernel); a launch with more takes the narrow layout
 constexpr int kWideClusters = 15;
@@ -227,7 +232,7 @@ __device__ __forceinline__ float part_weight(float m, float M) {
   return m == -INFINITY ? 0.f : (m == M ? 1.f : ex2(m - M));
 }
 
-template <int D, bool NARROW>
+template <int D, bool NARROW, bool PAIR>
 __global__ void __launch_bounds__(128, NARROW ? 3 : 2)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
                    const __grid_constant__ AttnArgs a) {
@@ -249,14 +254,25 @@ __global__ void __launch_bounds__(128, NARROW ? 3 : 2)
   uint64_t* bars = reinterpret_cast<uint64_t*>(s_x + 8);  // q, k (wide: and v), mma1, mma2, v
   uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 5);
   int* s_flag = reinterpret_cast<int*>(tslot + 1);
+  // pair: the second chunk's partial rows, received by the first chunk's CTA
+  float* p_o = reinterpret_cast<float*>((reinterpret_cast<uintptr_t>(s_flag + 4) + 15) &
+                                        ~static_cast<uintptr_t>(15));  // [8 rows][D]
+  float2* p_ml = reinterpret_cast<float2*>(p_o + 8 * D);  // [8 rows]
 
   const int tid = threadIdx.x, warp = tid >> 5;
-  const uint32_t rank = ptx::cluster_rank();
-  const int cl = (int)(blockIdx.x / kCluster), g = blockIdx.y;
+  // a cluster covers HALVES chunks of 8 tiles; half: this CTA's chunk of
+  // them, rank: its tile within the chunk
+  constexpr int HALVES = PAIR ? 2 : 1;
+  const uint32_t crank = ptx::cluster_rank();
+  const int half = (int)(crank >> 3);
+  const uint32_t rank = crank & 7u;
+  const int cl = (int)(blockIdx.x / (kCluster * HALVES)), g = blockIdx.y;
   int b = 0;
   while (b + 1 < a.rm.batch && a.cl_start[b + 1] <= cl) ++b;
   const int ci = cl - a.cl_start[b];
-  const int qt = ci / a.n_ch[b], c = ci - qt * a.n_ch[b];
+  const int ncl = (a.n_ch[b] + HALVES - 1) / HALVES;  // clusters per query tile
+  const int qt = ci / ncl, c2 = ci - qt * ncl;
+  const int c = c2 * HALVES + half;  // this CTA's chunk
   const int t = c * kCluster + (int)rank, p0 = t * kTile;
   const int r0 = a.rm.start[b], M = a.rm.start[b + 1] - r0;
   const int G = a.nq / a.nkv, qn = M * G;
@@ -266,7 +282,7 @@ __global__ void __launch_bounds__(128, NARROW ? 3 : 2)
   const int n_tiles = fits ? (kend + kTile - 1) / kTile : 0;
   const int n_chunks = (n_tiles + kCluster - 1) / kCluster;
   const bool active = t < n_tiles;      // this CTA's tile holds keys
-  const bool cl_active = c < n_chunks;  // uniform over the cluster
+  const bool cl_active = c2 * HALVES < n_chunks;  // uniform over the cluster
   if (!cl_active) return;               // the whole cluster holds no keys of this request
   const int z = (a.layer * a.batch + b) * a.nkv + g;
   const uint8_t* qsrc = a.qimg + ((size_t)(b * a.nkv + g) * a.qt_max + qt) * (size_t)Q_BYTES;
@@ -493,7 +509,7 @@ __global__ void __launch_bounds__(128, NARROW ? 3 : 2)
   // over its K image (every CTA's is consumed once all have arrived)
   ptx::cluster_wait();
   if (active) {
-    const uint32_t dst_rank = (uint32_t)(q >> 3), row = (uint32_t)(q & 7);
+    const uint32_t dst_rank = (uint32_t)(half * 8 + (q >> 3)), row = (uint32_t)(q & 7);
     if (pt == 0)
       dsmem_st_f2(ptx::dsmem_map(ptx::smem_u32(s_rml + rank * 8 + row), dst_rank), make_float2(m, l));
     if (m != -INFINITY) {
@@ -564,7 +580,48 @@ __global__ void __launch_bounds__(128, NARROW ? 3 : 2)
     }
   };
   if (n_chunks == 1) {
-    write_out(fo, fl);
+    if (half == 0) write_out(fo, fl);
+    return;
+  }
+  if (PAIR) {
+    // two chunks in this cluster: the second chunk's rows go to the CTA of
+    // the first chunk that holds the same rows, which folds the two in
+    // chunk order (the arithmetic of the fold over memory below)
+    if (half == 1) {
+      const uint32_t dst = ptx::dsmem_map(ptx::smem_u32(p_o + fj * D + fd), rank);
+#pragma unroll
+      for (int u = 0; u < DT / 4; ++u)
+        dsmem_st_f4(dst + 16u * u, make_float4(fo[4 * u], fo[4 * u + 1], fo[4 * u + 2], fo[4 * u + 3]));
+      if ((tid & 15) == 0)
+        dsmem_st_f2(ptx::dsmem_map(ptx::smem_u32(p_ml + fj), rank), make_float2(fm, fl));
+    }
+    ptx::cluster_sync();
+    if (half == 0) {
+      const float2 ml[2] = {make_float2(fm, fl), p_ml[fj]};
+      float cm = -INFINITY;
+#pragma unroll
+      for (int cc = 0; cc < 2; ++cc) cm = fmaxf(cm, ml[cc].x);
+      float cl_ = 0.f, co[DT];
+#pragma unroll
+      for (int e = 0; e < DT; ++e) co[e] = 0.f;
+#pragma unroll
+      for (int cc = 0; cc < 2; ++cc) {
+        const float w = part_weight(ml[cc].x, cm);
+        if (w != 0.f) {
+          cl_ += ml[cc].y * w;
+#pragma unroll
+          for (int u = 0; u < DT / 4; ++u) {
+            const float4 v = cc == 0 ? make_float4(fo[4 * u], fo[4 * u + 1], fo[4 * u + 2], fo[4 * u + 3])
+                                     : reinterpret_cast<const float4*>(p_o + fj * D + fd)[u];
+            co[4 * u + 0] += v.x * w;
+            co[4 * u + 1] += v.y * w;
+            co[4 * u + 2] += v.z * w;
+            co[4 * u + 3] += v.w * w;
+          }
+        }
+      }
+      write_out(co, cl_);
+    }
     return;
   }
   // ---- several chunks: this CTA's rows of the chunk partial go to memory;
@@ -638,28 +695,67 @@ __global__ void __launch_bounds__(128, NARROW ? 3 : 2)
   write_out(co, cl_);
 }
 
-template <int D, bool NARROW>
+// How many clusters of 16 of the pair kernel run at once (0 if none fits);
+// queried once per head size.
+template <int D>
+int pair_clusters_max() {
+  static const int n = [] {
+    constexpr uint32_t smem = attn_smem<false, true>();
+    if (cudaFuncSetAttribute(attn_tc_kernel<D, false, true>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess ||
+        cudaFuncSetAttribute(attn_tc_kernel<D, false, true>,
+                             cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess)
+      return 0;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(16 * 16, 1);
+    cfg.blockDim = dim3(128);
+    cfg.dynamicSmemBytes = smem;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = 16;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    int nc = 0;
+    if (cudaOccupancyMaxActiveClusters(&nc, attn_tc_kernel<D, false, true>, &cfg) != cudaSuccess) {
+      (void)cudaGetLastError();
+      return 0;
+    }
+    return nc;
+  }();
+  return n;
+}
+
+template <int D, bool NARROW, bool PAIR>
 cudaError_t launch_attn(const CUtensorMap& tk, const CUtensorMap& tv, const AttnArgs& a,
                         int clusters, cudaStream_t st) {
-  constexpr uint32_t smem = attn_smem<NARROW>();
+  constexpr uint32_t smem = attn_smem<NARROW, PAIR>();
+  constexpr int CL = PAIR ? 2 * kCluster : kCluster;
   static const cudaError_t attr = cudaFuncSetAttribute(
-      attn_tc_kernel<D, NARROW>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      attn_tc_kernel<D, NARROW, PAIR>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (attr != cudaSuccess) return attr;
+  // clusters of 16 are beyond the portable size of 8
+  static const cudaError_t attr16 =
+      PAIR ? cudaFuncSetAttribute(attn_tc_kernel<D, NARROW, PAIR>,
+                                  cudaFuncAttributeNonPortableClusterSizeAllowed, 1)
+           : cudaSuccess;
+  if (attr16 != cudaSuccess) return attr16;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(clusters * kCluster, a.nkv);
+  cfg.gridDim = dim3(clusters * CL, a.nkv);
   cfg.blockDim = dim3(128);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = st;
   cudaLaunchAttribute attr2[2];
   attr2[0].id = cudaLaunchAttributeClusterDimension;
-  attr2[0].val.clusterDim.x = kCluster;
+  attr2[0].val.clusterDim.x = CL;
   attr2[0].val.clusterDim.y = 1;
   attr2[0].val.clusterDim.z = 1;
   attr2[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr2[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr2;
   cfg.numAttrs = 2;
-  return cudaLaunchKernelEx(&cfg, attn_tc_kernel<D, NARROW>, tk, tv, a);
+  return cudaLaunchKernelEx(&cfg, attn_tc_kernel<D, NARROW, PAIR>, tk, tv, a);
 }
 
 }  // namespace
@@ -700,32 +796,47 @@ cudaError_t launch_attention_split(const RowMap& m, const Model& md, KvState& kv
   a.err = kv.d_err;
   a.timeout_ns = kv.wait_ns;
   const int G = c.n_q_heads / c.n_kv_heads;
-  a.cl_start[0] = 0;
+  int clusters8 = 0, max_nch = 0;
   for (int b = 0; b < kv.batch; ++b) {
     const int rows = m.start[b + 1] - m.start[b];
     const int64_t keys = kv.len_upper[b] + rows;
     int nch = (int)((keys + kChunk - 1) / kChunk);
     if (nch > kv.attn_chunks) nch = kv.attn_chunks;
     a.n_ch[b] = nch;
-    a.cl_start[b + 1] = a.cl_start[b] + attn_q_tiles(rows, G) * nch;
+    if (nch > max_nch) max_nch = nch;
+    clusters8 += attn_q_tiles(rows, G) * nch;
   }
+  // The same arithmetic whichever way the launch runs; the layout decides
+  // how many CTAs an SM holds and whether two chunks fold in one cluster.
+  // Narrow: more clusters of 8 than run at once.  Pair: every request has at
+  // most two chunks, and the clusters of 16 run at once.
+  const bool narrow = clusters8 * c.n_kv_heads > kWideClusters;
+  int clusters16 = 0;
+  for (int b = 0; b < kv.batch; ++b)
+    clusters16 += attn_q_tiles(m.start[b + 1] - m.start[b], G) * ((a.n_ch[b] + 1) / 2);
+  const int pair_max = c.head_dim == 128 ? pair_clusters_max<128>() : pair_clusters_max<64>();
+  const bool pair = !narrow && max_nch == 2 && clusters16 * c.n_kv_heads <= pair_max;
+  const int halves = pair ? 2 : 1;
+  a.cl_start[0] = 0;
+  for (int b = 0; b < kv.batch; ++b)
+    a.cl_start[b + 1] = a.cl_start[b] + attn_q_tiles(m.start[b + 1] - m.start[b], G) *
+                                            ((a.n_ch[b] + halves - 1) / halves);
   const int clusters = a.cl_start[kv.batch];
-  // the same arithmetic either way: the layout only decides how many CTAs an
-  // SM holds
-  const bool narrow = clusters * c.n_kv_heads > kWideClusters;
   const dim3 gf(m.rows, c.n_q_heads + 2 * c.n_kv_heads);
   cudaError_t e;
   kv.launches += 2;
   if (c.head_dim == 128) {
     e = launch_pdl(qkv_finish_kernel<128>, gf, dim3(64), 0, st, a);
     if (e == cudaSuccess)
-      e = narrow ? launch_attn<128, true>(kv.tm_kc, kv.tm_vc, a, clusters, st)
-                 : launch_attn<128, false>(kv.tm_kc, kv.tm_vc, a, clusters, st);
+      e = narrow ? launch_attn<128, true, false>(kv.tm_kc, kv.tm_vc, a, clusters, st)
+          : pair ? launch_attn<128, false, true>(kv.tm_kc, kv.tm_vc, a, clusters, st)
+                 : launch_attn<128, false, false>(kv.tm_kc, kv.tm_vc, a, clusters, st);
   } else {
     e = launch_pdl(qkv_finish_kernel<64>, gf, dim3(32), 0, st, a);
     if (e == cudaSuccess)
-      e = narrow ? launch_attn<64, true>(kv.tm_kc, kv.tm_vc, a, clusters, st)
-                 : launch_attn<64, false>(kv.tm_kc, kv.tm_vc, a, clusters, st);
+      e = narrow ? launch_attn<64, true, false>(kv.tm_kc, kv.tm_vc, a, clusters, st)
+          : pair ? launch_attn<64, false, true>(kv.tm_kc, kv.tm_vc, a, clusters, st)
+                 : launch_attn<64, false, false>(kv.tm_kc, kv.tm_vc, a, clusters, st);
   }
   return e;
 }
