@@ -556,9 +556,7 @@ as2d_status run_block(KvState& s, const int32_t* cand, const int32_t* k,
     LAUNCH(AS2D_KERNEL_QKV, tc_project(TC_PART, m, s, rm, m.w_qkv[l], s.tm_xn, m.qkv_rows, H, tp, st));
     LAUNCH(AS2D_KERNEL_ATTENTION, launch_attention_split(rm, m, s, l, st));
     tp.g_next = m.mlp_norm[l];
-    tp.small_ring = 1;
     LAUNCH(AS2D_KERNEL_O, tc_project(TC_RESID, m, s, rm, m.w_o[l], s.tm_ao, H, m.q_dim, tp, st));
-    tp.small_ring = 0;
     LAUNCH(AS2D_KERNEL_GATE_UP, tc_project(TC_SWIGLU, m, s, rm, m.w_gu[l], s.tm_xn, 2 * F, H, tp, st));
     tp.g_next = (l + 1 < c.n_layers) ? m.attn_norm[l + 1] : m.final_norm;
     LAUNCH(AS2D_KERNEL_DOWN, tc_project(TC_RESID, m, s, rm, m.w_down[l], s.tm_u, H, F, tp, st));
@@ -942,9 +940,7 @@ extern "C" as2d_status as2d_decode_step_static(as2d_model* mh, void* k_cache, vo
     LAUNCH(AS2D_KERNEL_QKV, tc_project(TC_PART, m, s, rm, m.w_qkv[l], s.tm_xn, m.qkv_rows, H, tp, st));
     LAUNCH(AS2D_KERNEL_ATTENTION, launch_attention_split(rm, m, s, l, st));
     tp.g_next = m.mlp_norm[l];
-    tp.small_ring = 1;
     LAUNCH(AS2D_KERNEL_O, tc_project(TC_RESID, m, s, rm, m.w_o[l], s.tm_ao, H, m.q_dim, tp, st));
-    tp.small_ring = 0;
     LAUNCH(AS2D_KERNEL_GATE_UP, tc_project(TC_SWIGLU, m, s, rm, m.w_gu[l], s.tm_xn, 2 * F, H, tp, st));
     tp.g_next = (l + 1 < c.n_layers) ? m.attn_norm[l + 1] : m.final_norm;
     LAUNCH(AS2D_KERNEL_DOWN, tc_project(TC_RESID, m, s, rm, m.w_down[l], s.tm_u, H, F, tp, st));

@@ -66,9 +66,6 @@ struct TcParams {
   int grid;              // CTAs
   int split;             // TC_PART: CTAs per tile (K split), else 0 (stream-K)
   int defer;             // stream-K: split tiles are finished by tc_reduce_kernel
-  int small_ring;        // a 5-deep ring (token rows <= 16), so that the CTA fits
-                         // on an SM beside an attention CTA and its first weight
-                         // tiles stream while the attention still runs
   float* part;           // TC_PART: [tile][split][part_ld][128] fp32 sums
   float* part_rinv;      // TC_PART: [part_ld] 1 / rms of each token row
   int part_ld;           // rows_alloc

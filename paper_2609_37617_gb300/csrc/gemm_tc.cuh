@@ -52,11 +52,9 @@ constexpr int tc_ring_depth(int nb) {
   return nb <= 32 ? AS2D_RING16 : nb <= 64 ? 5 : nb <= 96 ? 4 : nb <= 192 ? 3 : 2;
 }
 
-template <int NB, int RING = 0>
+template <int NB>
 struct TcShape {
-  // ring depth (RING: a shallower ring, so that a CTA fits on an SM beside
-  // an attention CTA)
-  static constexpr int S = RING ? RING : tc_ring_depth(NB);
+  static constexpr int S = tc_ring_depth(NB);  // weight-ring depth
   static constexpr uint32_t A_BYTES = 128 * 64 * 2;
   static constexpr uint32_t B_BYTES = NB * 64 * 2;   // one of the hi / lo operand tiles
   static constexpr uint32_t STAGE_B = 2 * B_BYTES;   // hi tile, then lo tile
@@ -347,10 +345,10 @@ __device__ __forceinline__ void tc_reduce_tile(const TcParams& p, float* sC, flo
   }
 }
 
-template <int NB, int EPI, int RING>
+template <int NB, int EPI>
 __global__ void __launch_bounds__(192, 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ TcParams p) {
-  using Sh = TcShape<NB, RING>;
+  using Sh = TcShape<NB>;
   constexpr int S = Sh::S;
   constexpr uint32_t A_BYTES = Sh::A_BYTES, B_BYTES = Sh::B_BYTES, STAGE_B = Sh::STAGE_B;
   constexpr int CH = Sh::CH, SP = Sh::SP;
@@ -660,15 +658,15 @@ __global__ void __launch_bounds__(128) tc_resid_finish_kernel(const __grid_const
   if (n == 0) p.ss[(size_t)tile * p.ss_ld + p.row0 + m] = ((red[0] + red[1]) + red[2]) + red[3];
 }
 
-template <int NB, int EPI, int RING = 0>
+template <int NB, int EPI>
 cudaError_t tc_gemm_launch(const CUtensorMap& x, const TcParams& p, cudaStream_t st) {
-  constexpr uint32_t smem = TcShape<NB, RING>::SMEM;
+  constexpr uint32_t smem = TcShape<NB>::SMEM;
   // set once per instantiation; a function-local static is initialised
   // exactly once even when several host threads launch at the same time
   static const cudaError_t attr = cudaFuncSetAttribute(
-      tc_gemm_kernel<NB, EPI, RING>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      tc_gemm_kernel<NB, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (attr != cudaSuccess) return attr;
-  cudaError_t e = launch_pdl(tc_gemm_kernel<NB, EPI, RING>, dim3(p.grid), dim3(192), smem, st, x, p);
+  cudaError_t e = launch_pdl(tc_gemm_kernel<NB, EPI>, dim3(p.grid), dim3(192), smem, st, x, p);
   if (e != cudaSuccess || !p.defer || p.grid < 2) return e;
   // only the residual projections leave their split tiles to a finishing kernel
   if (EPI != TC_RESID) return cudaErrorInvalidValue;
@@ -677,7 +675,6 @@ cudaError_t tc_gemm_launch(const CUtensorMap& x, const TcParams& p, cudaStream_t
 
 template <int EPI>
 cudaError_t tc_gemm_dispatch(int nb, const CUtensorMap& x, const TcParams& p, cudaStream_t st) {
-  if (EPI == TC_RESID && nb == 16 && p.small_ring) return tc_gemm_launch<16, EPI, 5>(x, p, st);
   switch (nb) {
     case 16: return tc_gemm_launch<16, EPI>(x, p, st);
     case 32: return tc_gemm_launch<32, EPI>(x, p, st);
