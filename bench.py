@@ -39,7 +39,7 @@ WORKLOAD = "7b"
 
 # dram__bytes_read.sum + dram__bytes_write.sum per launch from one ncu capture
 # of the kernel as it stands (profiles/); None once the kernel has changed.
-TRAFFIC = {"gate_up": 272226816}  # 271,882,752 read + 344,064 written
+TRAFFIC = {"gate_up": 272352000}  # 271,875,328 read + 476,672 written
 
 # Diagnostic legs that reuse the headline state (each rolls it back to L0 first).
 BUDGET_WIN, BUDGET_COMMIT, BUDGET_TRACES = 220, 180, 4
@@ -539,7 +539,8 @@ def run_ours(args, ws, rank, local):
                      "kernel_classes": "profiles/kernels_7b2l_k8_L1564.md",
                      "attention": "profiles/attention_7b2l_k8.md",
                      "gate_up": "profiles/gemm_gateup_7b_k8.md",
-                     "ragged": "profiles/kernels_7b2l_ragged16.md"},
+                     "ragged": "profiles/kernels_7b2l_ragged16.md",
+                     "1.5b": "profiles/kernels_1p5b_k8_L814.md"},
     }
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = guarded(errors, "cpu_baseline", cpu_baseline, args, cfg, L0, plans)
