@@ -217,6 +217,44 @@ def test_batch_of_requests_matches_single(pair):
     st.close()
 
 
+def test_attention_layouts_give_the_same_rows(pair):
+    """The attention runs a call in one of three layouts with the same
+    arithmetic: wide (one wave of clusters of 8), wide with clusters of 16
+    folding two 1024-key chunks in one cluster (every request of at most two
+    chunks), and narrow (several waves; V loaded over K).  A batch of four
+    requests of 1, 2, 3 and 4 chunks takes the narrow layout (20 clusters of 8
+    over the two kv heads); each request alone takes a wide one (the
+    two-chunk request: clusters of 16).  Every request's rows agree bit for
+    bit, and the two-chunk request matches the oracle."""
+    import torch
+    from synth import device as D
+    cfg = pair.cfg
+    lens = [1500, 3100, 300, 2600]
+    cap = 3200
+    roots = [int(t) for t in W.root_tokens(cfg, len(lens), 7)]
+    rng = np.random.default_rng(13)
+    cands = [[int(t) for t in rng.integers(0, cfg.vocab, k)] for k in (4, 2, 6, 0)]
+    st = pair.state(lens, cap, roots)
+    gpu = run_gpu_block(st, cfg, cands)
+    st.check()
+    starts = np.cumsum([0] + [len(c) + 1 for c in cands])
+    kc, vc = D.device_kv(cfg, lens, cap, pair.seed)
+    for b in range(len(lens)):
+        single = pair.state([lens[b]], cap, [roots[b]])
+        single.kc.copy_(kc[:, b:b + 1])
+        single.vc.copy_(vc[:, b:b + 1])
+        torch.cuda.synchronize()
+        g1 = run_gpu_block(single, cfg, [cands[b]])
+        single.check()
+        assert np.array_equal(g1[3], gpu[3][starts[b]:starts[b + 1]]), f"request {b}"
+        assert g1[0][0] == gpu[0][b] and g1[1][0] == gpu[1][b]
+        single.close()
+    oc = pair.oracle_cache(lens[0], cap, req=0)
+    ores = pair.oracle.verify_block(oc, lens[0], roots[0], cands[0])
+    compare_block(ores, gpu[3][0:5], gpu[2][0:5], gpu[0][0], gpu[1][0], 4)
+    st.close()
+
+
 def test_argument_and_device_errors(pair):
     import torch
     import paper_2609_37617_gb300 as lib
