@@ -211,17 +211,27 @@ __device__ __forceinline__ void dsmem_st_f2(uint32_t addr, float2 v) {
                : "memory");
 }
 
-// 64 columns of this thread's TMEM lane starting at `col`, into v.
-__device__ __forceinline__ void tmem_ld64(uint32_t taddr, float (&v)[64]) {
-  uint32_t a[32], b[32];
-  ptx::tmem_ld32(taddr, a);
-  ptx::tmem_ld32(taddr + 32, b);
+// 128 columns of this thread's TMEM lane starting at taddr: two loads, one
+// wait.
+__device__ __forceinline__ void tmem_ld128(uint32_t taddr, float (&v0)[64], float (&v1)[64]) {
+  uint32_t a[64], b[64];
+  ptx::tmem_ld_x64(taddr, a);
+  ptx::tmem_ld_x64(taddr + 64, b);
   ptx::tmem_ld_wait();
 #pragma unroll
-  for (int j = 0; j < 32; ++j) {
-    v[j] = __uint_as_float(a[j]);
-    v[32 + j] = __uint_as_float(b[j]);
+  for (int j = 0; j < 64; ++j) {
+    v0[j] = __uint_as_float(a[j]);
+    v1[j] = __uint_as_float(b[j]);
   }
+}
+
+// 64 columns of this thread's TMEM lane starting at `col`, into v.
+__device__ __forceinline__ void tmem_ld64(uint32_t taddr, float (&v)[64]) {
+  uint32_t a[64];
+  ptx::tmem_ld_x64(taddr, a);
+  ptx::tmem_ld_wait();
+#pragma unroll
+  for (int j = 0; j < 64; ++j) v[j] = __uint_as_float(a[j]);
 }
 
 // The weight of a part (max m) in a fold whose maximum is M: 2^(m - M), 0
@@ -370,7 +380,9 @@ __global__ void __launch_bounds__(128, NARROW ? 3 : 2)
   // Every thread arrives once at the split cluster barrier, when its CTA no
   // longer reads the image the cluster's partials are received into (the K
   // image: wide after the first product, narrow after the second, V being
-  // loaded there).  The others wait for the arrival only when they push.
+  // loaded there): the product's completion, observed on its mbarrier, means
+  // its operand reads are done, so the arrival needs no release.  The others
+  // wait for the arrival only when they push.
   if (active && ok) {
     if (tid == 0) {
       ptx::tc_fence_after();
@@ -387,7 +399,7 @@ __global__ void __launch_bounds__(128, NARROW ? 3 : 2)
     const bool ok1 = ptx::group_all(ptx::mbar_wait(&bars[2], 0, a.timeout_ns), 1, 128);
     // (after a timeout: once the product has drained)
     if (!ok1 && tid == 0) ptx::mbar_wait(&bars[2], 0, ptx::kDrainNs);
-    if (!NARROW || !ok1) ptx::cluster_arrive_release();
+    if (!NARROW || !ok1) ptx::cluster_arrive_relaxed();
     // narrow: the keys are consumed; V comes into their image during the softmax
     if (NARROW && ok1 && tid == 0) load_v();
     ptx::tc_fence_after();
@@ -398,8 +410,7 @@ __global__ void __launch_bounds__(128, NARROW ? 3 : 2)
       float sv[64];
       {
         float v0[64], v1[64];
-        tmem_ld64(tmem + lane_base, v0);
-        tmem_ld64(tmem + lane_base + 64, v1);
+        tmem_ld128(tmem + lane_base, v0, v1);
 #pragma unroll
         for (int j = 0; j < 64; ++j) {
           const float mine = pt ? v1[j] : v0[j], other = pt ? v0[j] : v1[j];
@@ -468,7 +479,7 @@ __global__ void __launch_bounds__(128, NARROW ? 3 : 2)
           ptx::mbar_wait(&bars[4], 0, ptx::kDrainNs);
           if (vok) ptx::mbar_wait(&bars[3], 0, ptx::kDrainNs);
         }
-        ptx::cluster_arrive_release();
+        ptx::cluster_arrive_relaxed();
       }
       ptx::tc_fence_after();
       if (ok2) {
@@ -497,7 +508,7 @@ __global__ void __launch_bounds__(128, NARROW ? 3 : 2)
       m = -INFINITY;  // nothing of this tile is passed on
     }
   } else {
-    ptx::cluster_arrive_release();  // no keys of this CTA's tile are read
+    ptx::cluster_arrive_relaxed();  // no keys of this CTA's tile are read
   }
   ptx::tc_fence_before();
   __syncthreads();
