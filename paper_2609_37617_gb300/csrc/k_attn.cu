@@ -185,8 +185,10 @@ __device__ __forceinline__ float ex2(float x) {
 // Values x[0..7] (>= 0) of columns e0..e0+7 (e0 % 8 == 0) of query q, as bf16
 // hi parts into row 2q and lo parts into row 2q + 1 of an operand image: hi =
 // x with its low 16 bits cleared (exact in bf16), lo = bf16(x - hi), so that
-// hi + lo matches x to about 17 bits.
-__device__ __forceinline__ void put_hilo8(uint8_t* img, int q, int e0, const float* x) {
+// hi + lo matches x to about 17 bits.  A thread of the odd half (pt = 1)
+// stores its lo row first: the two rows of one store instruction then cover
+// all eight 16-byte positions of the swizzle, not four.
+__device__ __forceinline__ void put_hilo8(uint8_t* img, int q, int pt, int e0, const float* x) {
   uint32_t hw[4], lw[4];
 #pragma unroll
   for (int u = 0; u < 4; ++u) {
@@ -196,8 +198,9 @@ __device__ __forceinline__ void put_hilo8(uint8_t* img, int q, int e0, const flo
                                                     x[2 * u + 1] - __uint_as_float(b1 & 0xFFFF0000u));
     lw[u] = *reinterpret_cast<const uint32_t*>(&lv);
   }
-  *reinterpret_cast<uint4*>(img + img_off(2 * q, e0)) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
-  *reinterpret_cast<uint4*>(img + img_off(2 * q + 1, e0)) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+  const uint4 h = make_uint4(hw[0], hw[1], hw[2], hw[3]), l = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+  *reinterpret_cast<uint4*>(img + img_off(2 * q + pt, e0)) = pt ? l : h;
+  *reinterpret_cast<uint4*>(img + img_off(2 * q + 1 - pt, e0)) = pt ? h : l;
 }
 
 __device__ __forceinline__ void dsmem_st_f4(uint32_t addr, float4 v) {
@@ -452,7 +455,7 @@ __global__ void __launch_bounds__(128, NARROW ? 3 : 2)
       l = pt ? lo_ + ls : ls + lo_;  // keys 0..63, then 64..127
       // P as bf16 hi (row 2q) and lo (row 2q + 1) parts, K-major by key
 #pragma unroll
-      for (int ch = 0; ch < 8; ++ch) put_hilo8(R0, q, 64 * pt + 8 * ch, sv + 8 * ch);
+      for (int ch = 0; ch < 8; ++ch) put_hilo8(R0, q, pt, 64 * pt + 8 * ch, sv + 8 * ch);
       if (NARROW) {
         vok = ptx::group_all(ptx::mbar_wait(&bars[4], 0, a.timeout_ns), 1, 128);
         if (vok) zero_v_tail();
