@@ -35,11 +35,17 @@
 //     keeping half of the dims;
 //   * the tile partials (m, l, O) are pushed through distributed shared
 //     memory to the CTA that folds their query rows (CTA r: rows 8r..8r+7),
-//     which folds the cluster's 8 tiles in tile order.  With one chunk the
-//     result is normalised and written (bf16 hi, lo); otherwise the CTA's rows
-//     of the chunk partial go to memory and the last CTA of those rows to
+//     which folds the chunk's 8 tiles in tile order.  With one chunk the
+//     result is normalised and written (bf16 hi, lo).  With two chunks in a
+//     cluster of 16 (PAIR), the second chunk's rows go to the first chunk's
+//     CTA of the same rows, which folds the two.  Otherwise the CTA's rows of
+//     the chunk partial go to memory and the last CTA of those rows to
 //     arrive, over the chunks of the (request, kv head, query tile), folds
 //     them in chunk order.
+// Shared-memory layouts (the same arithmetic): wide, K and V in their own
+// images, two CTAs per SM; NARROW, V loaded over K once the first product is
+// done and O accumulated over S in TMEM, three CTAs per SM, for launches of
+// several waves of clusters.
 // Every fold boundary is a fixed absolute key position (128-key tiles,
 // 1024-key chunks), and a fold with a part a row cannot see (fully masked:
 // m = -inf, l = 0, O = 0) leaves it bitwise unchanged, so a row's result does
