@@ -340,9 +340,6 @@ __global__ void __launch_bounds__(128, NARROW ? 3 : 2)
     load_kv();
   }
   ptx::griddep_wait();
-  // every CTA of this grid holds its TMEM by now: the next kernel (the O
-  // projection) may start and stream its first weight tiles meanwhile
-  ptx::griddep_launch_dependents();
   if (tid == 0 && active) {
     if (!early) load_kv();
     ptx::mbar_arrive_expect_tx(&bars[0], Q_BYTES);
@@ -363,6 +360,9 @@ __global__ void __launch_bounds__(128, NARROW ? 3 : 2)
   if (active) {
     ok = ptx::mbar_wait(&bars[0], 0, a.timeout_ns) && ptx::mbar_wait(&bars[1], 0, a.timeout_ns);
     ok = ptx::group_all(ok, 1, 128);
+    // the tile has arrived: the next kernel (the O projection) may start and
+    // stream its first weight tiles now, without delaying these loads
+    ptx::griddep_launch_dependents();
     if (!ok) {
       if (tid == 0) {
         atomicOr(a.err, kErrTimeout);
@@ -373,6 +373,7 @@ __global__ void __launch_bounds__(128, NARROW ? 3 : 2)
       __syncthreads();
     }
   }
+  if (!active) ptx::griddep_launch_dependents();
   // values past the call's last key (stale entries, or NaN in a poisoned
   // cache) would reach O through 0 * V: those rows of the V tile are zeroed
   auto zero_v_tail = [&]() {
