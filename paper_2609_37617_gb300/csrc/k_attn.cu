@@ -360,9 +360,6 @@ __global__ void __launch_bounds__(128, NARROW ? 3 : 2)
   if (active) {
     ok = ptx::mbar_wait(&bars[0], 0, a.timeout_ns) && ptx::mbar_wait(&bars[1], 0, a.timeout_ns);
     ok = ptx::group_all(ok, 1, 128);
-    // the tile has arrived: the next kernel (the O projection) may start and
-    // stream its first weight tiles now, without delaying these loads
-    ptx::griddep_launch_dependents();
     if (!ok) {
       if (tid == 0) {
         atomicOr(a.err, kErrTimeout);
@@ -373,7 +370,6 @@ __global__ void __launch_bounds__(128, NARROW ? 3 : 2)
       __syncthreads();
     }
   }
-  if (!active) ptx::griddep_launch_dependents();
   // values past the call's last key (stale entries, or NaN in a poisoned
   // cache) would reach O through 0 * V: those rows of the V tile are zeroed
   auto zero_v_tail = [&]() {
@@ -520,6 +516,10 @@ __global__ void __launch_bounds__(128, NARROW ? 3 : 2)
   } else {
     ptx::cluster_arrive_relaxed();  // no keys of this CTA's tile are read
   }
+  // the tile's products are done: the next kernel (the O projection) may
+  // start and stream its first weight tiles now (earlier, they would compete
+  // with this kernel's own loads)
+  ptx::griddep_launch_dependents();
   ptx::tc_fence_before();
   __syncthreads();
   if (warp == 0) ptx::tmem_dealloc(tmem, TMEM_COLS);
