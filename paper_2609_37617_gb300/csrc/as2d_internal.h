@@ -65,7 +65,7 @@ struct TcParams {
   long long units;       // n_tiles * kb
   int grid;              // CTAs
   int split;             // TC_PART: CTAs per tile (K split), else 0 (stream-K)
-  int defer;             // stream-K: split tiles are finished by tc_reduce_kernel
+  int defer;             // stream-K: split tiles are finished by tc_resid_finish_kernel
   float* part;           // TC_PART: [tile][split][part_ld][128] fp32 sums
   float* part_rinv;      // TC_PART: [part_ld] 1 / rms of each token row
   int part_ld;           // rows_alloc
