@@ -456,9 +456,36 @@ __global__ void __launch_bounds__(128, NARROW ? 3 : 2)
       const float ls = (ls4[0] + ls4[1]) + (ls4[2] + ls4[3]);
       const float lo_ = __shfl_xor_sync(0xFFFFFFFFu, ls, 1);
       l = pt ? lo_ + ls : ls + lo_;  // keys 0..63, then 64..127
-      // P as bf16 hi (row 2q) and lo (row 2q + 1) parts, K-major by key
+      // P as bf16 hi (row 2q) and lo (row 2q + 1) parts: hi = P with its low
+      // 16 bits cleared, lo = bf16(P - hi).  Wide: into TMEM over S (the
+      // second product's A operand, lane 2q + pt its row, two keys per
+      // column), each lane completing its row with the partner's half of the
+      // keys.  Narrow: into the operand image in shared memory, K-major by key.
+      if (!NARROW) {
+        uint32_t hw[32], lw[32], row[64];
 #pragma unroll
-      for (int ch = 0; ch < 8; ++ch) put_hilo8(R0, q, pt, 64 * pt + 8 * ch, sv + 8 * ch);
+        for (int j = 0; j < 32; ++j) {
+          const uint32_t b0 = __float_as_uint(sv[2 * j]), b1 = __float_as_uint(sv[2 * j + 1]);
+          hw[j] = (b0 >> 16) | (b1 & 0xFFFF0000u);
+          const __nv_bfloat162 lv =
+              __floats2bfloat162_rn(sv[2 * j] - __uint_as_float(b0 & 0xFFFF0000u),
+                                    sv[2 * j + 1] - __uint_as_float(b1 & 0xFFFF0000u));
+          lw[j] = *reinterpret_cast<const uint32_t*>(&lv);
+        }
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+          // the hi lane takes the partner's hi words (keys 64..127), the lo
+          // lane the partner's lo words (keys 0..63)
+          const uint32_t got = __shfl_xor_sync(0xFFFFFFFFu, pt ? hw[j] : lw[j], 1);
+          row[j] = pt ? got : hw[j];
+          row[32 + j] = pt ? lw[j] : got;
+        }
+        ptx::tmem_st_x64(tmem + lane_base, row);
+        ptx::tmem_st_wait();
+      } else {
+#pragma unroll
+        for (int ch = 0; ch < 8; ++ch) put_hilo8(R0, q, pt, 64 * pt + 8 * ch, sv + 8 * ch);
+      }
       if (NARROW) {
         vok = ptx::group_all(ptx::mbar_wait(&bars[4], 0, a.timeout_ns), 1, 128);
         if (vok) zero_v_tail();
@@ -472,9 +499,14 @@ __global__ void __launch_bounds__(128, NARROW ? 3 : 2)
         constexpr uint32_t IDESC2 = ptx::idesc_bf16_f32(128, D, true);
 #pragma unroll
         for (int kk = 0; kk < kTile / 16; ++kk) {
-          const uint64_t ad = ptx::sdesc_sw128(ptx::smem_u32(R0 + (kk >> 2) * kRegion)) + 2 * (kk & 3);
           const uint64_t bd = ptx::sdesc_sw128_mn(ptx::smem_u32(R2) + kk * 2048u, kRegion, 1024u);
-          ptx::mma_bf16(tmem + (NARROW ? 0 : 128), ad, bd, IDESC2, kk > 0 ? 1u : 0u);
+          if (NARROW) {
+            const uint64_t ad = ptx::sdesc_sw128(ptx::smem_u32(R0 + (kk >> 2) * kRegion)) + 2 * (kk & 3);
+            ptx::mma_bf16(tmem, ad, bd, IDESC2, kk > 0 ? 1u : 0u);
+          } else {
+            // A: 16 keys = 8 columns per k-step
+            ptx::mma_bf16_ta(tmem + 128, tmem + 8u * kk, bd, IDESC2, kk > 0 ? 1u : 0u);
+          }
         }
         ptx::mma_commit(&bars[3]);
       }
