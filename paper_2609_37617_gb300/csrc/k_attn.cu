@@ -75,9 +75,11 @@ constexpr uint32_t attn_smem() {
 }
 static_assert(3 * (attn_smem<true, false>() + 1024) <= 228 * 1024, "three narrow CTAs per SM");
 static_assert(2 * (attn_smem<false, true>() + 1024) <= 228 * 1024, "two wide CTAs per SM");
-// at most this many clusters of 8 run at once (cudaOccupancyMaxActiveClusters
-// of the wide kernel); a launch with more takes the narrow layout
-constexpr int kWideClusters = 15;
+// A launch of more clusters of 8 than this takes the narrow layout.  The wide
+// kernel's shared memory allows 36 clusters of 8 at two CTAs per SM (the
+// occupancy calculator reports 15); measured on 7B and 1.5B calls, the wide
+// layout is the faster up to 28 clusters and much the slower at 36.
+constexpr int kWideClusters = 28;
 
 struct AttnArgs {
   RowMap rm;

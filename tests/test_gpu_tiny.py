@@ -221,19 +221,19 @@ def test_attention_layouts_give_the_same_rows(pair):
     """The attention runs a call in one of three layouts with the same
     arithmetic: wide (one wave of clusters of 8), wide with clusters of 16
     folding two 1024-key chunks in one cluster (every request of at most two
-    chunks), and narrow (several waves; V loaded over K).  A batch of four
-    requests of 1, 2, 3 and 4 chunks takes the narrow layout (20 clusters of 8
-    over the two kv heads); each request alone takes a wide one (the
-    two-chunk request: clusters of 16).  Every request's rows agree bit for
-    bit, and the two-chunk request matches the oracle."""
+    chunks), and narrow (several waves; V loaded over K).  A batch of six
+    requests of 2, 4, 1, 3, 4 and 4 chunks takes the narrow layout (36
+    clusters of 8 over the two kv heads); each request alone takes a wide
+    one (the two-chunk request: clusters of 16).  Every request's rows agree
+    bit for bit, and the two-chunk request matches the oracle."""
     import torch
     from synth import device as D
     cfg = pair.cfg
-    lens = [1500, 3100, 300, 2600]
-    cap = 3200
+    lens = [1500, 3100, 300, 2600, 4000, 3900]
+    cap = 4100
     roots = [int(t) for t in W.root_tokens(cfg, len(lens), 7)]
     rng = np.random.default_rng(13)
-    cands = [[int(t) for t in rng.integers(0, cfg.vocab, k)] for k in (4, 2, 6, 0)]
+    cands = [[int(t) for t in rng.integers(0, cfg.vocab, k)] for k in (4, 2, 6, 0, 3, 5)]
     st = pair.state(lens, cap, roots)
     gpu = run_gpu_block(st, cfg, cands)
     st.check()
