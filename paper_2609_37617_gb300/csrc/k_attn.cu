@@ -45,7 +45,7 @@
 // Shared-memory layouts (the same arithmetic): wide, K and V in their own
 // images, two CTAs per SM; NARROW, V loaded over K once the first product is
 // done and O accumulated over S in TMEM, three CTAs per SM, for launches of
-// several waves of clusters.
+// more clusters than the wide layout serves well.
 // Every fold boundary is a fixed absolute key position (128-key tiles,
 // 1024-key chunks), and a fold with a part a row cannot see (fully masked:
 // m = -inf, l = 0, O = 0) leaves it bitwise unchanged, so a row's result does
@@ -61,10 +61,10 @@ constexpr int kCluster = 8;   // CTAs per cluster
 constexpr int kChunk = kTile * kCluster;
 constexpr int kQT = 64;       // queries per query tile (hi and lo rows interleaved)
 constexpr uint32_t kRegion = 128 * 128;  // one 64-column region of 128 rows, bytes
-// Shared memory: the Q / P image, then the K and V tiles.  Wide (one wave of
-// clusters): K and V in separate images, both requested at the start.
-// Narrow (launches of several waves): V is loaded over K once the first
-// product has consumed it, so that three CTAs fit on an SM.
+// Shared memory: the Q / P image, then the K and V tiles.  Wide (launches of
+// up to kWideClusters clusters of 8): K and V in separate images, both
+// requested at the start.  Narrow (larger launches): V is loaded over K once
+// the first product has consumed it, so that three CTAs fit on an SM.
 // Pair (wide only): clusters of 16 CTAs, two chunks, whose second chunk's
 // partial comes to the first chunk's CTAs through distributed shared memory
 // ([8 rows][d] floats and [8] (max, sum)) instead of through global memory.
@@ -863,8 +863,8 @@ cudaError_t launch_attention_split(const RowMap& m, const Model& md, KvState& kv
   }
   // The same arithmetic whichever way the launch runs; the layout decides
   // how many CTAs an SM holds and whether two chunks fold in one cluster.
-  // Narrow: more clusters of 8 than run at once.  Pair: every request has at
-  // most two chunks, and the clusters of 16 run at once.
+  // Narrow: more than kWideClusters clusters of 8.  Pair: every request has
+  // at most two chunks, and the clusters of 16 run at once.
   const bool narrow = clusters8 * c.n_kv_heads > kWideClusters;
   int clusters16 = 0;
   for (int b = 0; b < kv.batch; ++b)
