@@ -37,11 +37,11 @@
 //     memory to the CTA that folds their query rows (CTA r: rows 8r..8r+7),
 //     which folds the chunk's 8 tiles in tile order.  With one chunk the
 //     result is normalised and written (bf16 hi, lo).  With two chunks in a
-//     cluster of 16 (PAIR), the second chunk's rows go to the first chunk's
-//     CTA of the same rows, which folds the two.  Otherwise the CTA's rows of
-//     the chunk partial go to memory and the last CTA of those rows to
-//     arrive, over the chunks of the (request, kv head, query tile), folds
-//     them in chunk order.
+//     cluster of 16 (PAIR), CTA r receives rows 4r..4r+3 from all 16 tiles
+//     and folds each chunk's tiles, then the two chunks.  Otherwise the
+//     CTA's rows of the chunk partial go to memory and the last CTA of those
+//     rows to arrive, over the chunks of the (request, kv head, query tile),
+//     folds them in chunk order.
 // Shared-memory layouts (the same arithmetic): wide, K and V in their own
 // images, two CTAs per SM; NARROW, V loaded over K once the first product is
 // done and O accumulated over S in TMEM, three CTAs per SM, for launches of
@@ -65,13 +65,12 @@ constexpr uint32_t kRegion = 128 * 128;  // one 64-column region of 128 rows, by
 // up to kWideClusters clusters of 8): K and V in separate images, both
 // requested at the start.  Narrow (larger launches): V is loaded over K once
 // the first product has consumed it, so that three CTAs fit on an SM.
-// Pair (wide only): clusters of 16 CTAs, two chunks, whose second chunk's
-// partial comes to the first chunk's CTAs through distributed shared memory
-// ([8 rows][d] floats and [8] (max, sum)) instead of through global memory.
+// Pair (wide only): clusters of 16 CTAs over two chunks, each CTA folding 4
+// query rows of both, so that the chunks fold without going through global
+// memory.
 template <bool NARROW, bool PAIR>
 constexpr uint32_t attn_smem() {
-  return (NARROW ? 2 : 3) * 32768 + 64 * 8 + 8 * 4 + 5 * 8 + 16 +
-         (PAIR ? 16 + 8 * 128 * 4 + 8 * 8 : 0) + 1024;
+  return (NARROW ? 2 : 3) * 32768 + 64 * 8 + 8 * 4 + 5 * 8 + 16 + 1024;
 }
 static_assert(3 * (attn_smem<true, false>() + 1024) <= 228 * 1024, "three narrow CTAs per SM");
 static_assert(2 * (attn_smem<false, true>() + 1024) <= 228 * 1024, "two wide CTAs per SM");
@@ -253,6 +252,39 @@ __device__ __forceinline__ float part_weight(float m, float M) {
   return m == -INFINITY ? 0.f : (m == M ? 1.f : ex2(m - M));
 }
 
+// Dims [fd, fd + DT) of row fr of query tile qt, normalised (o / l), as
+// bf16 hi and lo parts into the attention output; rows past the call's
+// queries are skipped.
+template <int D, int DT>
+__device__ __forceinline__ void write_rows(const AttnArgs& a, const float* o_, float Ls, int fr,
+                                           int fd, int qt, int qn, int G, int g, int r0) {
+  const int fqg = qt * kQT + fr;
+  if (fqg >= qn) return;
+  const int i = fqg / G, hq = g * G + (fqg - i * G);
+  const size_t at = (size_t)(r0 + i) * a.nq * D + (size_t)hq * D + fd;
+  uint32_t hw[DT / 2], lw[DT / 2];
+#pragma unroll
+  for (int e = 0; e < DT / 2; ++e) {
+    const float v0 = o_[2 * e] / Ls, v1 = o_[2 * e + 1] / Ls;
+    const __nv_bfloat162 hv = __floats2bfloat162_rn(v0, v1);
+    const float2 hf = __bfloat1622float2(hv);
+    const __nv_bfloat162 lv = __floats2bfloat162_rn(v0 - hf.x, v1 - hf.y);
+    hw[e] = *reinterpret_cast<const uint32_t*>(&hv);
+    lw[e] = *reinterpret_cast<const uint32_t*>(&lv);
+  }
+#pragma unroll
+  for (int u = 0; u < DT / 8; ++u) {
+    *reinterpret_cast<uint4*>(a.ao + at + 8 * u) =
+        make_uint4(hw[4 * u], hw[4 * u + 1], hw[4 * u + 2], hw[4 * u + 3]);
+    *reinterpret_cast<uint4*>(a.ao + (size_t)a.lo_row * a.nq * D + at + 8 * u) =
+        make_uint4(lw[4 * u], lw[4 * u + 1], lw[4 * u + 2], lw[4 * u + 3]);
+  }
+  if (DT % 8) {  // four dims
+    *reinterpret_cast<uint2*>(a.ao + at) = make_uint2(hw[0], hw[1]);
+    *reinterpret_cast<uint2*>(a.ao + (size_t)a.lo_row * a.nq * D + at) = make_uint2(lw[0], lw[1]);
+  }
+}
+
 template <int D, bool NARROW, bool PAIR>
 __global__ void __launch_bounds__(128, NARROW ? 3 : 2)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
@@ -270,15 +302,12 @@ __global__ void __launch_bounds__(128, NARROW ? 3 : 2)
   uint8_t* R1 = sm + 32768;    // K tile -> the partials received from the cluster
   uint8_t* R2 = NARROW ? R1 : sm + 65536;  // V tile (narrow: over K, after the first product)
   float* recv = reinterpret_cast<float*>(R1);  // [8 tiles][8 rows][D] received
-  float2* s_rml = reinterpret_cast<float2*>(sm + (NARROW ? 2 : 3) * 32768);  // [8][8] (max, sum)
+  // [tiles of the cluster][rows folded here] (max, sum): [8][8], pair [16][4]
+  float2* s_rml = reinterpret_cast<float2*>(sm + (NARROW ? 2 : 3) * 32768);
   float* s_x = reinterpret_cast<float*>(s_rml + 64);      // [8] scratch
   uint64_t* bars = reinterpret_cast<uint64_t*>(s_x + 8);  // q, k (wide: and v), mma1, mma2, v
   uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 5);
   int* s_flag = reinterpret_cast<int*>(tslot + 1);
-  // pair: the second chunk's partial rows, received by the first chunk's CTA
-  float* p_o = reinterpret_cast<float*>((reinterpret_cast<uintptr_t>(s_flag + 4) + 15) &
-                                        ~static_cast<uintptr_t>(15));  // [8 rows][D]
-  float2* p_ml = reinterpret_cast<float2*>(p_o + 8 * D);  // [8 rows]
 
   const int tid = threadIdx.x, warp = tid >> 5;
   // a cluster covers HALVES chunks of 8 tiles; half: this CTA's chunk of
@@ -559,23 +588,85 @@ __global__ void __launch_bounds__(128, NARROW ? 3 : 2)
   if (warp == 0) ptx::tmem_dealloc(tmem, TMEM_COLS);
 
   // ---- the cluster's tile partials, pushed to the CTA that folds them ----
-  // CTA r folds query rows 8r..8r+7; it receives, from every CTA i of the
-  // cluster, rows (max, sum) into s_rml[i][row] and O into recv[i][row][d],
-  // over its K image (every CTA's is consumed once all have arrived)
+  // CTA r folds query rows RPC r .. RPC r + RPC - 1 (RPC: 8 in a cluster of
+  // 8, 4 in a cluster of 16); it receives, from the CTA of every tile i of
+  // the cluster, rows (max, sum) into s_rml[i][row] and O into
+  // recv[i][row][d], over its K image (every CTA's is consumed once all have
+  // arrived)
+  constexpr int RPC = PAIR ? 4 : 8;
   ptx::cluster_wait();
   if (active) {
-    const uint32_t dst_rank = (uint32_t)(half * 8 + (q >> 3)), row = (uint32_t)(q & 7);
+    const uint32_t dst_rank = (uint32_t)(q / RPC), row = (uint32_t)(q % RPC);
     if (pt == 0)
-      dsmem_st_f2(ptx::dsmem_map(ptx::smem_u32(s_rml + rank * 8 + row), dst_rank), make_float2(m, l));
+      dsmem_st_f2(ptx::dsmem_map(ptx::smem_u32(s_rml + crank * RPC + row), dst_rank), make_float2(m, l));
     if (m != -INFINITY) {
       const uint32_t dst =
-          ptx::dsmem_map(ptx::smem_u32(recv + (rank * 8 + row) * D + pt * DH), dst_rank);
+          ptx::dsmem_map(ptx::smem_u32(recv + (crank * RPC + row) * D + pt * DH), dst_rank);
 #pragma unroll
       for (int u = 0; u < DH / 4; ++u)
         dsmem_st_f4(dst + 16u * u, make_float4(o[4 * u], o[4 * u + 1], o[4 * u + 2], o[4 * u + 3]));
     }
   }
   ptx::cluster_sync();
+
+  if (PAIR) {
+    // ---- two chunks in one cluster: CTA r folds rows 4r..4r+3, each
+    // chunk's 8 tiles in tile order, then the two chunk partials in chunk
+    // order: the arithmetic of the one-chunk fold and of the fold through
+    // memory below (thread: row fj, dims [fd, fd + 4))
+    constexpr int TPR = D / 4 < 32 ? D / 4 : 32;  // threads per row
+    if (tid < 4 * TPR) {
+      const int fj = tid / TPR, fr = 4 * (int)crank + fj, fd = 4 * (tid % TPR);
+      float cmx[2], cls[2], cfo[2][4];
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const int nh = min(kCluster, n_tiles - (c2 * 2 + h) * kCluster);  // may be <= 0
+        float fm = -INFINITY;
+        float2 pml[kCluster];
+#pragma unroll
+        for (int i = 0; i < kCluster; ++i) {
+          pml[i] = (i < nh) ? s_rml[(h * kCluster + i) * 4 + fj] : make_float2(-INFINITY, 0.f);
+          fm = fmaxf(fm, pml[i].x);
+        }
+        float fl = 0.f, fo[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int i = 0; i < kCluster; ++i) {
+          const float w = part_weight(pml[i].x, fm);
+          if (w != 0.f) {
+            fl += pml[i].y * w;
+            const float4 v = *reinterpret_cast<const float4*>(recv + ((h * kCluster + i) * 4 + fj) * D + fd);
+            fo[0] += v.x * w;
+            fo[1] += v.y * w;
+            fo[2] += v.z * w;
+            fo[3] += v.w * w;
+          }
+        }
+        cmx[h] = fm;
+        cls[h] = fl;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) cfo[h][e] = fo[e];
+      }
+      if (n_chunks == 1) {
+        write_rows<D, 4>(a, cfo[0], cls[0], fr, fd, qt, qn, G, g, r0);
+      } else {
+        float cm = -INFINITY;
+#pragma unroll
+        for (int cc = 0; cc < 2; ++cc) cm = fmaxf(cm, cmx[cc]);
+        float cl_ = 0.f, co[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int cc = 0; cc < 2; ++cc) {
+          const float w = part_weight(cmx[cc], cm);
+          if (w != 0.f) {
+            cl_ += cls[cc] * w;
+#pragma unroll
+            for (int e = 0; e < 4; ++e) co[e] += cfo[cc][e] * w;
+          }
+        }
+        write_rows<D, 4>(a, co, cl_, fr, fd, qt, qn, G, g, r0);
+      }
+    }
+    return;
+  }
 
   // ---- fold (thread: query row 8 rank + fj, dims [fd, fd + DT)) ----------
   const int n_here = min(kCluster, n_tiles - c * kCluster);  // tiles of this chunk with keys
@@ -608,75 +699,10 @@ __global__ void __launch_bounds__(128, NARROW ? 3 : 2)
   }
   // normalise and write the row's dims (o / l as bf16 hi, lo)
   auto write_out = [&](const float* o_, float Ls) {
-    const int fqg = qt * kQT + fr;
-    if (fqg >= qn) return;
-    const int i = fqg / G, hq = g * G + (fqg - i * G);
-    const size_t at = (size_t)(r0 + i) * a.nq * D + (size_t)hq * D + fd;
-    uint32_t hw[DT / 2], lw[DT / 2];
-#pragma unroll
-    for (int e = 0; e < DT / 2; ++e) {
-      const float v0 = o_[2 * e] / Ls, v1 = o_[2 * e + 1] / Ls;
-      const __nv_bfloat162 hv = __floats2bfloat162_rn(v0, v1);
-      const float2 hf = __bfloat1622float2(hv);
-      const __nv_bfloat162 lv = __floats2bfloat162_rn(v0 - hf.x, v1 - hf.y);
-      hw[e] = *reinterpret_cast<const uint32_t*>(&hv);
-      lw[e] = *reinterpret_cast<const uint32_t*>(&lv);
-    }
-#pragma unroll
-    for (int u = 0; u < DT / 8; ++u) {
-      *reinterpret_cast<uint4*>(a.ao + at + 8 * u) =
-          make_uint4(hw[4 * u], hw[4 * u + 1], hw[4 * u + 2], hw[4 * u + 3]);
-      *reinterpret_cast<uint4*>(a.ao + (size_t)a.lo_row * a.nq * D + at + 8 * u) =
-          make_uint4(lw[4 * u], lw[4 * u + 1], lw[4 * u + 2], lw[4 * u + 3]);
-    }
-    if (DT % 8) {  // D = 64: four dims
-      *reinterpret_cast<uint2*>(a.ao + at) = make_uint2(hw[0], hw[1]);
-      *reinterpret_cast<uint2*>(a.ao + (size_t)a.lo_row * a.nq * D + at) = make_uint2(lw[0], lw[1]);
-    }
+    write_rows<D, DT>(a, o_, Ls, fr, fd, qt, qn, G, g, r0);
   };
   if (n_chunks == 1) {
-    if (half == 0) write_out(fo, fl);
-    return;
-  }
-  if (PAIR) {
-    // two chunks in this cluster: the second chunk's rows go to the CTA of
-    // the first chunk that holds the same rows, which folds the two in
-    // chunk order (the arithmetic of the fold over memory below)
-    if (half == 1) {
-      const uint32_t dst = ptx::dsmem_map(ptx::smem_u32(p_o + fj * D + fd), rank);
-#pragma unroll
-      for (int u = 0; u < DT / 4; ++u)
-        dsmem_st_f4(dst + 16u * u, make_float4(fo[4 * u], fo[4 * u + 1], fo[4 * u + 2], fo[4 * u + 3]));
-      if ((tid & 15) == 0)
-        dsmem_st_f2(ptx::dsmem_map(ptx::smem_u32(p_ml + fj), rank), make_float2(fm, fl));
-    }
-    ptx::cluster_sync();
-    if (half == 0) {
-      const float2 ml[2] = {make_float2(fm, fl), p_ml[fj]};
-      float cm = -INFINITY;
-#pragma unroll
-      for (int cc = 0; cc < 2; ++cc) cm = fmaxf(cm, ml[cc].x);
-      float cl_ = 0.f, co[DT];
-#pragma unroll
-      for (int e = 0; e < DT; ++e) co[e] = 0.f;
-#pragma unroll
-      for (int cc = 0; cc < 2; ++cc) {
-        const float w = part_weight(ml[cc].x, cm);
-        if (w != 0.f) {
-          cl_ += ml[cc].y * w;
-#pragma unroll
-          for (int u = 0; u < DT / 4; ++u) {
-            const float4 v = cc == 0 ? make_float4(fo[4 * u], fo[4 * u + 1], fo[4 * u + 2], fo[4 * u + 3])
-                                     : reinterpret_cast<const float4*>(p_o + fj * D + fd)[u];
-            co[4 * u + 0] += v.x * w;
-            co[4 * u + 1] += v.y * w;
-            co[4 * u + 2] += v.z * w;
-            co[4 * u + 3] += v.w * w;
-          }
-        }
-      }
-      write_out(co, cl_);
-    }
+    write_out(fo, fl);
     return;
   }
   // ---- several chunks: this CTA's rows of the chunk partial go to memory;
