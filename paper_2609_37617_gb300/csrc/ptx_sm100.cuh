@@ -103,6 +103,15 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* m, uin
 // 3D tiled load: box at coordinates (x = innermost, y, z), completion counted
 // in bytes on `bar`; x * element size must be a multiple of 16 bytes.  Parts
 // of the box outside the tensor are filled with zeros.
+// Prefetch one box of a 3D tensor map into L2 (no completion to wait for;
+// the parts of the box outside the tensor are skipped).
+__device__ __forceinline__ void tma_prefetch_3d(const CUtensorMap* m, int32_t x, int32_t y, int32_t z) {
+  asm volatile("cp.async.bulk.prefetch.tensor.3d.L2.global.tile [%0, {%1, %2, %3}];" ::"l"(
+                   reinterpret_cast<uint64_t>(m)),
+               "r"(x), "r"(y), "r"(z)
+               : "memory");
+}
+
 __device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* m, uint64_t* bar,
                                             int32_t x, int32_t y, int32_t z, uint64_t policy) {
   asm volatile(
