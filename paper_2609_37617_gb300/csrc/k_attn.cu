@@ -61,6 +61,10 @@ constexpr int kCluster = 8;   // CTAs per cluster
 constexpr int kChunk = kTile * kCluster;
 constexpr int kQT = 64;       // queries per query tile (hi and lo rows interleaved)
 constexpr uint32_t kRegion = 128 * 128;  // one 64-column region of 128 rows, bytes
+// chunks whose partial rows the last arriver stages in shared memory: [15][8
+// rows][128] floats and [15][8] (max, sum) within the first two 32 KB images
+constexpr int kStage = 15;
+static_assert(kStage * 8 * 128 * 4 + kStage * 8 * 8 <= 2 * 32768, "staging fits two images");
 // Shared memory: the Q / P image, then the K and V tiles.  Wide (launches of
 // up to kWideClusters clusters of 8): K and V in separate images, both
 // requested at the start.  Narrow (larger launches): V is loaded over K once
@@ -738,6 +742,44 @@ __global__ void __launch_bounds__(128, NARROW ? 3 : 2)
   float cl_ = 0.f, co[DT];
 #pragma unroll
   for (int e = 0; e < DT; ++e) co[e] = 0.f;
+  if (n_chunks > 8 && n_chunks <= kStage) {
+    // nine or more chunks: every chunk's rows come into shared memory (over
+    // the Q / P and K images, no longer read) by copies issued together, one
+    // memory round trip instead of two through registers
+    float* st_o = reinterpret_cast<float*>(sm);                          // [chunk][8 rows][D]
+    float2* st_ml = reinterpret_cast<float2*>(sm + kStage * 8 * D * 4);  // [chunk][8 rows]
+    for (int cc = 0; cc < n_chunks; ++cc) {
+      const size_t pc = item * a.chunks_max + cc;
+      const float* src = a.ws_o + (pc * kQT + fr) * D + fd;
+      float* dst = st_o + (cc * 8 + fj) * D + fd;
+#pragma unroll
+      for (int u = 0; u < DT / 4; ++u) ptx::cp_async16(dst + 4 * u, src + 4 * u);
+      // (max, sum) of rows fj and fj + 1 in one copy
+      if ((tid & 15) == 0 && (fj & 1) == 0) ptx::cp_async16(st_ml + cc * 8 + fj, a.ws_ml + pc * kQT + fr);
+    }
+    ptx::cp_async_wait_all();
+    __syncthreads();
+    float cm = -INFINITY;
+    for (int cc = 0; cc < n_chunks; ++cc) cm = fmaxf(cm, st_ml[cc * 8 + fj].x);
+    for (int cc = 0; cc < n_chunks; ++cc) {
+      const float2 ml = st_ml[cc * 8 + fj];
+      const float w = part_weight(ml.x, cm);
+      if (w != 0.f) {
+        cl_ += ml.y * w;
+        const float4* src = reinterpret_cast<const float4*>(st_o + (cc * 8 + fj) * D + fd);
+#pragma unroll
+        for (int u = 0; u < DT / 4; ++u) {
+          const float4 v = src[u];
+          co[4 * u + 0] += v.x * w;
+          co[4 * u + 1] += v.y * w;
+          co[4 * u + 2] += v.z * w;
+          co[4 * u + 3] += v.w * w;
+        }
+      }
+    }
+    write_out(co, cl_);
+    return;
+  }
   // eight chunks' values in flight at a time; the first eight are requested
   // together with every chunk's maximum, so that up to eight chunks take one
   // memory round trip

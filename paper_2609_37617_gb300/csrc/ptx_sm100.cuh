@@ -103,6 +103,17 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* m, uin
 // 3D tiled load: box at coordinates (x = innermost, y, z), completion counted
 // in bytes on `bar`; x * element size must be a multiple of 16 bytes.  Parts
 // of the box outside the tensor are filled with zeros.
+// 16-byte asynchronous copy global -> shared (L2 only), and the wait for all
+// of the thread's outstanding copies.
+__device__ __forceinline__ void cp_async16(void* smem_dst, const void* gmem_src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(smem_dst)),
+               "l"(__cvta_generic_to_global(gmem_src))
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
+}
+
 // Prefetch one box of a 3D tensor map into L2 (no completion to wait for;
 // the parts of the box outside the tensor are skipped).
 __device__ __forceinline__ void tma_prefetch_3d(const CUtensorMap* m, int32_t x, int32_t y, int32_t z) {
