@@ -30,9 +30,10 @@
 //     added by a shuffle, each lane keeping half of the keys; masking (causal,
 //     and keys past the call's end) and P = 2^(S - m) with the tile's own
 //     maximum m and sum l;
-//   * O = P V on tcgen05 (P's hi and lo rows interleaved the same way; B = V
-//     read MN-major from the TMA image); hi + lo added by a shuffle, each lane
-//     keeping half of the dims;
+//   * O = P V on tcgen05 (P's hi and lo rows interleaved the same way, as
+//     the A operand in TMEM over S, or in the narrow layout as a shared-memory
+//     image over Q; B = V read MN-major from the TMA image); hi + lo added by
+//     a shuffle, each lane keeping half of the dims;
 //   * the tile partials (m, l, O) are pushed through distributed shared
 //     memory to the CTA that folds their query rows (CTA r: rows 8r..8r+7),
 //     which folds the chunk's 8 tiles in tile order.  With one chunk the
@@ -41,11 +42,12 @@
 //     and folds each chunk's tiles, then the two chunks.  Otherwise the
 //     CTA's rows of the chunk partial go to memory and the last CTA of those
 //     rows to arrive, over the chunks of the (request, kv head, query tile),
-//     folds them in chunk order.
+//     folds them in chunk order (9 to 15 chunks staged in shared memory).
 // Shared-memory layouts (the same arithmetic): wide, K and V in their own
 // images, two CTAs per SM; NARROW, V loaded over K once the first product is
-// done and O accumulated over S in TMEM, three CTAs per SM, for launches of
-// more clusters than the wide layout serves well.
+// done (from L2, where the launch is small enough to prefetch it) and O
+// accumulated over S in TMEM, three CTAs per SM, for launches of more
+// clusters than the wide layout serves well.
 // Every fold boundary is a fixed absolute key position (128-key tiles,
 // 1024-key chunks), and a fold with a part a row cannot see (fully masked:
 // m = -inf, l = 0, O = 0) leaves it bitwise unchanged, so a row's result does
