@@ -826,8 +826,13 @@ __global__ void __launch_bounds__(128, NARROW ? 3 : 2)
   write_out(co, cl_);
 }
 
-// How many clusters of 16 of the pair kernel run at once (0 if none fits);
-// queried once per head size.
+// Clusters of 16 resident at once, two CTAs per SM: 14 in a residency probe
+// (the occupancy calculator reports 7).
+constexpr int kPairClusters = 14;
+
+// How many clusters of 16 of the pair kernel the occupancy calculator allows
+// (0 if none fits, or the launch attributes are refused); queried once per
+// head size.
 template <int D>
 int pair_clusters_max() {
   static const int n = [] {
@@ -949,8 +954,9 @@ cudaError_t launch_attention_split(const RowMap& m, const Model& md, KvState& kv
   int clusters16 = 0;
   for (int b = 0; b < kv.batch; ++b)
     clusters16 += attn_q_tiles(m.start[b + 1] - m.start[b], G) * ((a.n_ch[b] + 1) / 2);
-  const int pair_max = c.head_dim == 128 ? pair_clusters_max<128>() : pair_clusters_max<64>();
-  const bool pair = !narrow && max_nch == 2 && clusters16 * c.n_kv_heads <= pair_max;
+  const bool pair_fits =
+      (c.head_dim == 128 ? pair_clusters_max<128>() : pair_clusters_max<64>()) > 0;
+  const bool pair = !narrow && pair_fits && max_nch == 2 && clusters16 * c.n_kv_heads <= kPairClusters;
   const int halves = pair ? 2 : 1;
   a.cl_start[0] = 0;
   for (int b = 0; b < kv.batch; ++b)
