@@ -83,8 +83,8 @@ static_assert(2 * (attn_smem<false, true>() + 1024) <= 228 * 1024, "two wide CTA
 // A launch of more clusters of 8 than this takes the narrow layout.  The wide
 // kernel's shared memory allows 36 clusters of 8 at two CTAs per SM (the
 // occupancy calculator reports 15); measured on 7B and 1.5B calls, the wide
-// layout is the faster up to 28 clusters and much the slower at 36.
-constexpr int kWideClusters = 28;
+// layout is the faster up to 32 clusters and much the slower at 36.
+constexpr int kWideClusters = 32;
 
 struct AttnArgs {
   RowMap rm;
