@@ -778,6 +778,7 @@ def run_e2e(args, lib, W, state, traj, plans, cfg, L0, root0, sh, stream):
     cand_d = torch.zeros(k, dtype=torch.int32, device="cuda")
     out_d = torch.zeros(2, dtype=torch.int32, device="cuda")
     steps = min(args.steps, len(plans))
+    out = lib.make_verify_out(out_d.data_ptr(), out_d.data_ptr() + 4)
     m = 0
     committed = 0
     torch.cuda.synchronize()
@@ -785,7 +786,6 @@ def run_e2e(args, lib, W, state, traj, plans, cfg, L0, root0, sh, stream):
     for i in range(steps):
         cand_h.numpy()[:] = W.apply_plan(traj_h[m + 1:m + 1 + k], plans[i], cfg.vocab)
         cand_d.copy_(cand_h, non_blocking=True)
-        out = lib.make_verify_out(out_d.data_ptr(), out_d.data_ptr() + 4)
         lib._check(lib.as2d_verify_block(state.handle, cand_d.data_ptr(), [k], out, sh),
                    "as2d_verify_block")
         out_h.copy_(out_d, non_blocking=True)
