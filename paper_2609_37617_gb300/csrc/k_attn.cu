@@ -85,6 +85,9 @@ static_assert(2 * (attn_smem<false, true>() + 1024) <= 228 * 1024, "two wide CTA
 // occupancy calculator reports 15); measured on 7B and 1.5B calls, the wide
 // layout is the faster up to 32 clusters and much the slower at 36.
 constexpr int kWideClusters = 32;
+// clusters of 8 the narrow layout keeps resident (three CTAs per SM, residency
+// probe); larger launches take four CTAs per SM
+constexpr int kNarrowClusters = 51;
 
 struct AttnArgs {
   RowMap rm;
@@ -259,6 +262,45 @@ __device__ __forceinline__ float part_weight(float m, float M) {
   return m == -INFINITY ? 0.f : (m == M ? 1.f : ex2(m - M));
 }
 
+// The tile's scores of this thread's 64 keys kb .. kb + 63 (hi + lo, in sv)
+// -> P = 2^(S - m) in sv (visible keys: key <= lim; a masked key gets 0,
+// never -inf), with the tile's maximum m and sum l over both halves of the
+// keys (the partner lane holds the other half).
+__device__ __forceinline__ void softmax_tail(float (&sv)[64], int pt, int kb, int lim, float& m,
+                                             float& l) {
+  // a half-tile wholly at or below the row's limit needs no mask
+  const bool all_vis = kb + 63 <= lim;
+  float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+  if (all_vis) {
+#pragma unroll
+    for (int j = 0; j < 64; ++j) mx4[j & 3] = fmaxf(mx4[j & 3], sv[j]);
+  } else {
+#pragma unroll
+    for (int j = 0; j < 64; ++j)
+      if (kb + j <= lim) mx4[j & 3] = fmaxf(mx4[j & 3], sv[j]);
+  }
+  const float mx = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3]));
+  m = fmaxf(mx, __shfl_xor_sync(0xFFFFFFFFu, mx, 1));
+  // sums in four interleaved parts, then ((0 + 1) + (2 + 3)): a fixed order
+  float ls4[4] = {0.f, 0.f, 0.f, 0.f};
+  if (all_vis) {
+#pragma unroll
+    for (int j = 0; j < 64; ++j) {
+      sv[j] = ex2(sv[j] - m);
+      ls4[j & 3] += sv[j];
+    }
+  } else {
+#pragma unroll
+    for (int j = 0; j < 64; ++j) {
+      sv[j] = (kb + j <= lim) ? ex2(sv[j] - m) : 0.f;
+      ls4[j & 3] += sv[j];
+    }
+  }
+  const float ls = (ls4[0] + ls4[1]) + (ls4[2] + ls4[3]);
+  const float lo_ = __shfl_xor_sync(0xFFFFFFFFu, ls, 1);
+  l = pt ? lo_ + ls : ls + lo_;  // keys 0..63, then 64..127
+}
+
 // Dims [fd, fd + DT) of row fr of query tile qt, normalised (o / l), as
 // bf16 hi and lo parts into the attention output; rows past the call's
 // queries are skipped.
@@ -292,6 +334,166 @@ __device__ __forceinline__ void write_rows(const AttnArgs& a, const float* o_, f
   }
 }
 
+// The fold of a chunk's 8 tile partials for query rows 8 rank .. 8 rank + 7
+// (received into s_rml [8 tiles][8 rows] and recv [8 tiles][8 rows][D]) and
+// what follows it: with one chunk the rows are normalised and written; with
+// several, the rows of the chunk partial go to memory and the last CTA of
+// these rows to arrive folds the chunks in chunk order (9 to stage_max chunks
+// staged in shared memory at sm, whose images are no longer read).
+template <int D>
+__device__ __forceinline__ void fold_chunk8(const AttnArgs& a, const float* recv,
+                                            const float2* s_rml, int* s_flag, uint8_t* sm,
+                                            int stage_max, uint32_t rank, int c, int n_tiles,
+                                            int n_chunks, int b, int g, int qt, int qn, int G,
+                                            int r0) {
+  constexpr int DT = D / 16;  // dims per thread (8 rows x 16 threads)
+  const int tid = threadIdx.x;
+  // ---- fold (thread: query row 8 rank + fj, dims [fd, fd + DT)) ----------
+  const int n_here = min(kCluster, n_tiles - c * kCluster);  // tiles of this chunk with keys
+  const int fj = tid >> 4, fr = 8 * (int)rank + fj, fd = DT * (tid & 15);
+  float fm = -INFINITY;
+  float2 pml[kCluster];
+#pragma unroll
+  for (int i = 0; i < kCluster; ++i) {
+    pml[i] = (i < n_here) ? s_rml[i * 8 + fj] : make_float2(-INFINITY, 0.f);
+    fm = fmaxf(fm, pml[i].x);
+  }
+  float fl = 0.f, fo[DT];
+#pragma unroll
+  for (int e = 0; e < DT; ++e) fo[e] = 0.f;
+#pragma unroll
+  for (int i = 0; i < kCluster; ++i) {
+    const float w = part_weight(pml[i].x, fm);
+    if (w != 0.f) {
+      fl += pml[i].y * w;
+      const float4* src = reinterpret_cast<const float4*>(recv + (i * 8 + fj) * D + fd);
+#pragma unroll
+      for (int u = 0; u < DT / 4; ++u) {
+        const float4 v = src[u];
+        fo[4 * u + 0] += v.x * w;
+        fo[4 * u + 1] += v.y * w;
+        fo[4 * u + 2] += v.z * w;
+        fo[4 * u + 3] += v.w * w;
+      }
+    }
+  }
+  // normalise and write the row's dims (o / l as bf16 hi, lo)
+  auto write_out = [&](const float* o_, float Ls) {
+    write_rows<D, DT>(a, o_, Ls, fr, fd, qt, qn, G, g, r0);
+  };
+  if (n_chunks == 1) {
+    write_out(fo, fl);
+    return;
+  }
+  // ---- several chunks: this CTA's rows of the chunk partial go to memory;
+  // the last chunk's CTA of these rows to arrive folds them in chunk order
+  const size_t item = (size_t)(b * a.nkv + g) * a.qt_max + qt;
+  {
+    const size_t pc = item * a.chunks_max + c;
+    float4* dst = reinterpret_cast<float4*>(a.ws_o + (pc * kQT + fr) * D + fd);
+#pragma unroll
+    for (int u = 0; u < DT / 4; ++u)
+      dst[u] = make_float4(fo[4 * u], fo[4 * u + 1], fo[4 * u + 2], fo[4 * u + 3]);
+    if ((tid & 15) == 0) a.ws_ml[pc * kQT + fr] = make_float2(fm, fl);
+  }
+  __syncthreads();
+  int* cnt = a.cnt + item * kCluster + rank;
+  if (tid == 0) {
+    // the arrival releases the CTA's writes above (ordered before it by the
+    // barrier) and acquires the other chunks' partials for the last arriver
+    int prev;
+    asm volatile("atom.add.acq_rel.gpu.s32 %0, [%1], 1;" : "=r"(prev) : "l"(cnt) : "memory");
+    const int last = prev == n_chunks - 1;
+    if (last) *cnt = 0;  // every chunk of these rows has arrived
+    *s_flag = last;
+  }
+  __syncthreads();
+  if (!*s_flag) return;
+  float cl_ = 0.f, co[DT];
+#pragma unroll
+  for (int e = 0; e < DT; ++e) co[e] = 0.f;
+  if (n_chunks > 8 && n_chunks <= stage_max) {
+    // nine or more chunks: every chunk's rows come into shared memory (over
+    // the Q / P and K images, no longer read) by copies issued together, one
+    // memory round trip instead of two through registers
+    float* st_o = reinterpret_cast<float*>(sm);                          // [chunk][8 rows][D]
+    float2* st_ml = reinterpret_cast<float2*>(sm + stage_max * 8 * D * 4);  // [chunk][8 rows]
+    for (int cc = 0; cc < n_chunks; ++cc) {
+      const size_t pc = item * a.chunks_max + cc;
+      const float* src = a.ws_o + (pc * kQT + fr) * D + fd;
+      float* dst = st_o + (cc * 8 + fj) * D + fd;
+#pragma unroll
+      for (int u = 0; u < DT / 4; ++u) ptx::cp_async16(dst + 4 * u, src + 4 * u);
+      // (max, sum) of rows fj and fj + 1 in one copy
+      if ((tid & 15) == 0 && (fj & 1) == 0) ptx::cp_async16(st_ml + cc * 8 + fj, a.ws_ml + pc * kQT + fr);
+    }
+    ptx::cp_async_wait_all();
+    __syncthreads();
+    float cm = -INFINITY;
+    for (int cc = 0; cc < n_chunks; ++cc) cm = fmaxf(cm, st_ml[cc * 8 + fj].x);
+    for (int cc = 0; cc < n_chunks; ++cc) {
+      const float2 ml = st_ml[cc * 8 + fj];
+      const float w = part_weight(ml.x, cm);
+      if (w != 0.f) {
+        cl_ += ml.y * w;
+        const float4* src = reinterpret_cast<const float4*>(st_o + (cc * 8 + fj) * D + fd);
+#pragma unroll
+        for (int u = 0; u < DT / 4; ++u) {
+          const float4 v = src[u];
+          co[4 * u + 0] += v.x * w;
+          co[4 * u + 1] += v.y * w;
+          co[4 * u + 2] += v.z * w;
+          co[4 * u + 3] += v.w * w;
+        }
+      }
+    }
+    write_out(co, cl_);
+    return;
+  }
+  // eight chunks' values in flight at a time; the first eight are requested
+  // together with every chunk's maximum, so that up to eight chunks take one
+  // memory round trip
+  float4 v[8][DT / 4];
+  float2 ml[8];
+  auto load8 = [&](int c0) {
+#pragma unroll
+    for (int u8 = 0; u8 < 8; ++u8)
+      if (c0 + u8 < n_chunks) {
+        const size_t pc = item * a.chunks_max + c0 + u8;
+        ml[u8] = __ldcg(a.ws_ml + pc * kQT + fr);
+        const float4* src = reinterpret_cast<const float4*>(a.ws_o + (pc * kQT + fr) * D + fd);
+#pragma unroll
+        for (int u = 0; u < DT / 4; ++u) v[u8][u] = __ldcg(src + u);
+      }
+  };
+  load8(0);
+  float cm = -INFINITY;
+  for (int cc = 8; cc < n_chunks; ++cc)
+    cm = fmaxf(cm, __ldcg(a.ws_ml + (item * a.chunks_max + cc) * kQT + fr).x);
+#pragma unroll
+  for (int u8 = 0; u8 < 8; ++u8)
+    if (u8 < n_chunks) cm = fmaxf(cm, ml[u8].x);
+  for (int c0 = 0; c0 < n_chunks; c0 += 8) {
+    if (c0 > 0) load8(c0);
+#pragma unroll
+    for (int u8 = 0; u8 < 8; ++u8)
+      if (c0 + u8 < n_chunks) {
+        const float w = part_weight(ml[u8].x, cm);
+        if (w != 0.f) {
+          cl_ += ml[u8].y * w;
+#pragma unroll
+          for (int u = 0; u < DT / 4; ++u) {
+            co[4 * u + 0] += v[u8][u].x * w;
+            co[4 * u + 1] += v[u8][u].y * w;
+            co[4 * u + 2] += v[u8][u].z * w;
+            co[4 * u + 3] += v[u8][u].w * w;
+          }
+        }
+      }
+  }
+  write_out(co, cl_);
+}
+
 template <int D, bool NARROW, bool PAIR>
 __global__ void __launch_bounds__(128, NARROW ? 3 : 2)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
@@ -301,7 +503,6 @@ __global__ void __launch_bounds__(128, NARROW ? 3 : 2)
   constexpr uint32_t TMEM_COLS = NARROW ? 128 : 256;   // narrow: O over S
   constexpr uint32_t Q_BYTES = 2u * kQT * D * 2;
   constexpr int DH = D / 2;           // dims each thread of a hi/lo pair keeps
-  constexpr int DT = D / 16;          // dims per thread in the folds (8 rows x 16 threads)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -466,39 +667,7 @@ __global__ void __launch_bounds__(128, NARROW ? 3 : 2)
           sv[j] = mine + __shfl_xor_sync(0xFFFFFFFFu, other, 1);
         }
       }
-      const int kb = p0 + 64 * pt;
-      // keys at or below the row's limit are visible; a half-tile wholly
-      // below it needs no mask (masked keys are skipped, never given -inf)
-      const bool all_vis = kb + 63 <= lim;
-      float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-      if (all_vis) {
-#pragma unroll
-        for (int j = 0; j < 64; ++j) mx4[j & 3] = fmaxf(mx4[j & 3], sv[j]);
-      } else {
-#pragma unroll
-        for (int j = 0; j < 64; ++j)
-          if (kb + j <= lim) mx4[j & 3] = fmaxf(mx4[j & 3], sv[j]);
-      }
-      const float mx = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3]));
-      m = fmaxf(mx, __shfl_xor_sync(0xFFFFFFFFu, mx, 1));
-      // sums in four interleaved parts, then ((0 + 1) + (2 + 3)): a fixed order
-      float ls4[4] = {0.f, 0.f, 0.f, 0.f};
-      if (all_vis) {
-#pragma unroll
-        for (int j = 0; j < 64; ++j) {
-          sv[j] = ex2(sv[j] - m);
-          ls4[j & 3] += sv[j];
-        }
-      } else {
-#pragma unroll
-        for (int j = 0; j < 64; ++j) {
-          sv[j] = (kb + j <= lim) ? ex2(sv[j] - m) : 0.f;
-          ls4[j & 3] += sv[j];
-        }
-      }
-      const float ls = (ls4[0] + ls4[1]) + (ls4[2] + ls4[3]);
-      const float lo_ = __shfl_xor_sync(0xFFFFFFFFu, ls, 1);
-      l = pt ? lo_ + ls : ls + lo_;  // keys 0..63, then 64..127
+      softmax_tail(sv, pt, p0 + 64 * pt, lim, m, l);
       // P as bf16 hi (row 2q) and lo (row 2q + 1) parts: hi = P with its low
       // 16 bits cleared, lo = bf16(P - hi).  Wide: into TMEM over S (the
       // second product's A operand, lane 2q + pt its row, two keys per
@@ -680,150 +849,280 @@ __global__ void __launch_bounds__(128, NARROW ? 3 : 2)
     return;
   }
 
-  // ---- fold (thread: query row 8 rank + fj, dims [fd, fd + DT)) ----------
-  const int n_here = min(kCluster, n_tiles - c * kCluster);  // tiles of this chunk with keys
-  const int fj = tid >> 4, fr = 8 * (int)rank + fj, fd = DT * (tid & 15);
-  float fm = -INFINITY;
-  float2 pml[kCluster];
-#pragma unroll
-  for (int i = 0; i < kCluster; ++i) {
-    pml[i] = (i < n_here) ? s_rml[i * 8 + fj] : make_float2(-INFINITY, 0.f);
-    fm = fmaxf(fm, pml[i].x);
-  }
-  float fl = 0.f, fo[DT];
-#pragma unroll
-  for (int e = 0; e < DT; ++e) fo[e] = 0.f;
-#pragma unroll
-  for (int i = 0; i < kCluster; ++i) {
-    const float w = part_weight(pml[i].x, fm);
-    if (w != 0.f) {
-      fl += pml[i].y * w;
-      const float4* src = reinterpret_cast<const float4*>(recv + (i * 8 + fj) * D + fd);
-#pragma unroll
-      for (int u = 0; u < DT / 4; ++u) {
-        const float4 v = src[u];
-        fo[4 * u + 0] += v.x * w;
-        fo[4 * u + 1] += v.y * w;
-        fo[4 * u + 2] += v.z * w;
-        fo[4 * u + 3] += v.w * w;
-      }
-    }
-  }
-  // normalise and write the row's dims (o / l as bf16 hi, lo)
-  auto write_out = [&](const float* o_, float Ls) {
-    write_rows<D, DT>(a, o_, Ls, fr, fd, qt, qn, G, g, r0);
-  };
-  if (n_chunks == 1) {
-    write_out(fo, fl);
-    return;
-  }
-  // ---- several chunks: this CTA's rows of the chunk partial go to memory;
-  // the last chunk's CTA of these rows to arrive folds them in chunk order
-  const size_t item = (size_t)(b * a.nkv + g) * a.qt_max + qt;
-  {
-    const size_t pc = item * a.chunks_max + c;
-    float4* dst = reinterpret_cast<float4*>(a.ws_o + (pc * kQT + fr) * D + fd);
-#pragma unroll
-    for (int u = 0; u < DT / 4; ++u)
-      dst[u] = make_float4(fo[4 * u], fo[4 * u + 1], fo[4 * u + 2], fo[4 * u + 3]);
-    if ((tid & 15) == 0) a.ws_ml[pc * kQT + fr] = make_float2(fm, fl);
-  }
-  __syncthreads();
-  int* cnt = a.cnt + item * kCluster + rank;
+  fold_chunk8<D>(a, recv, s_rml, s_flag, sm, kStage, rank, c, n_tiles, n_chunks, b, g, qt, qn, G,
+                 r0);
+}
+
+// Four CTAs per SM (QUAD), for launches of more clusters than the narrow
+// layout keeps resident: the narrow layout's tiles, arithmetic and fold in
+// 48 KB of shared memory, 128 TMEM columns and at most 128 registers a
+// thread.  The first product runs in halves of d (the whole Q image, one
+// 16 KB region of the K tile at a time); V is loaded over Q; P goes to TMEM
+// over S, and the second product runs in 64-dim halves of O over S's second
+// half, each read out before the next.  S is read and P written in 16-key
+// chunks, so that no thread holds a whole row of either.
+constexpr uint32_t attn4_smem() { return 32768 + 16384 + 64 * 8 + 8 * 8 + 4 + 16 + 1024; }
+static_assert(4 * (attn4_smem() + 1024) <= 228 * 1024, "four CTAs per SM");
+// chunks the last arriver stages in shared memory: [11][8 rows][128] floats
+// and [11][8] (max, sum) within the Q and K images
+constexpr int kStage4 = 11;
+static_assert(kStage4 * 8 * 128 * 4 + kStage4 * 8 * 8 <= 32768 + 16384, "staging fits");
+
+template <int D>
+__global__ void __launch_bounds__(128, 4)
+    attn_tc4_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
+                    const __grid_constant__ AttnArgs a) {
+  constexpr int NR = D / 64;          // 64-column regions of a K / V tile
+  constexpr uint32_t Q_BYTES = 2u * kQT * D * 2;
+  constexpr int DH = D / 2;           // dims each thread of a hi/lo pair keeps
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* sm = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  uint8_t* R0 = sm;            // Q image -> V tile -> the partials received from the cluster
+  uint8_t* RK = sm + 32768;    // one 64-column region of the K tile
+  float* recv = reinterpret_cast<float*>(R0);                // [8 tiles][8 rows][D]
+  float2* s_rml = reinterpret_cast<float2*>(sm + 49152);    // [8][8] (max, sum)
+  uint64_t* bars = reinterpret_cast<uint64_t*>(s_rml + 64);  // q, k0, s0, k1, s1, v, o0, o1
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 8);
+  int* s_flag = reinterpret_cast<int*>(tslot + 1);
+
+  const int tid = threadIdx.x, warp = tid >> 5;
+  const uint32_t rank = ptx::cluster_rank();
+  const int cl = (int)(blockIdx.x / kCluster), g = blockIdx.y;
+  int b = 0;
+  while (b + 1 < a.rm.batch && a.cl_start[b + 1] <= cl) ++b;
+  const int ci = cl - a.cl_start[b];
+  const int ncl = a.n_ch[b];  // clusters per query tile
+  const int qt = ci / ncl, c = ci - qt * ncl;
+  const int t = c * kCluster + (int)rank, p0 = t * kTile;
+  const int r0 = a.rm.start[b], M = a.rm.start[b + 1] - r0;
+  const int G = a.nq / a.nkv, qn = M * G;
+  const int L = a.len[b];
+  const bool fits = rows_fit(L, M, a.cap);
+  const int kend = L + M;
+  const int n_tiles = fits ? (kend + kTile - 1) / kTile : 0;
+  const int n_chunks = (n_tiles + kCluster - 1) / kCluster;
+  const bool active = t < n_tiles;
+  if (c >= n_chunks) return;  // the whole cluster holds no keys of this request
+  const int z = (a.layer * a.batch + b) * a.nkv + g;
+  const uint8_t* qsrc = a.qimg + ((size_t)(b * a.nkv + g) * a.qt_max + qt) * (size_t)Q_BYTES;
+
   if (tid == 0) {
-    // the arrival releases the CTA's writes above (ordered before it by the
-    // barrier) and acquires the other chunks' partials for the last arriver
-    int prev;
-    asm volatile("atom.add.acq_rel.gpu.s32 %0, [%1], 1;" : "=r"(prev) : "l"(cnt) : "memory");
-    const int last = prev == n_chunks - 1;
-    if (last) *cnt = 0;  // every chunk of these rows has arrived
-    *s_flag = last;
+    for (int i = 0; i < 8; ++i) ptx::mbar_init(&bars[i], 1);
+    ptx::fence_mbar_init();
   }
+  if (warp == 0) ptx::tmem_alloc(tslot, 128);
+  ptx::tc_fence_before();
   __syncthreads();
-  if (!*s_flag) return;
-  float cl_ = 0.f, co[DT];
+  ptx::tc_fence_after();
+  const uint32_t tmem = *tslot;
+  const uint32_t lane_base = (uint32_t)(32 * warp) << 16;
+
+  const uint64_t pol = ptx::policy_evict_first();
+  uint32_t issued = 0;  // (thread 0) barriers with a copy or product outstanding
+  auto load_k = [&](int h, int bar) {  // region h of the K tile into RK
+    ptx::mbar_arrive_expect_tx(&bars[bar], kRegion);
+    ptx::tma_load_3d(RK, &tmK, &bars[bar], 64 * h, p0, z, pol);
+    issued |= 1u << bar;
+  };
+  auto prefetch_rest = [&]() {  // the other K regions and V, into L2
 #pragma unroll
-  for (int e = 0; e < DT; ++e) co[e] = 0.f;
-  if (n_chunks > 8 && n_chunks <= kStage) {
-    // nine or more chunks: every chunk's rows come into shared memory (over
-    // the Q / P and K images, no longer read) by copies issued together, one
-    // memory round trip instead of two through registers
-    float* st_o = reinterpret_cast<float*>(sm);                          // [chunk][8 rows][D]
-    float2* st_ml = reinterpret_cast<float2*>(sm + kStage * 8 * D * 4);  // [chunk][8 rows]
-    for (int cc = 0; cc < n_chunks; ++cc) {
-      const size_t pc = item * a.chunks_max + cc;
-      const float* src = a.ws_o + (pc * kQT + fr) * D + fd;
-      float* dst = st_o + (cc * 8 + fj) * D + fd;
+    for (int h = 1; h < NR; ++h) ptx::tma_prefetch_3d(&tmK, 64 * h, p0, z);
 #pragma unroll
-      for (int u = 0; u < DT / 4; ++u) ptx::cp_async16(dst + 4 * u, src + 4 * u);
-      // (max, sum) of rows fj and fj + 1 in one copy
-      if ((tid & 15) == 0 && (fj & 1) == 0) ptx::cp_async16(st_ml + cc * 8 + fj, a.ws_ml + pc * kQT + fr);
+    for (int h = 0; h < NR; ++h) ptx::tma_prefetch_3d(&tmV, 64 * h, p0, z);
+  };
+  // a tile of entries older than this call does not depend on the finishing
+  // kernel: request it before the wait
+  const bool early = active && p0 + kTile <= L;
+  if (tid == 0 && early) {
+    ptx::prefetch_tmap(&tmK);
+    ptx::prefetch_tmap(&tmV);
+    load_k(0, 1);
+    prefetch_rest();
+  }
+  ptx::griddep_wait();
+  if (tid == 0 && active) {
+    if (!early) {
+      load_k(0, 1);
+      prefetch_rest();
     }
-    ptx::cp_async_wait_all();
-    __syncthreads();
-    float cm = -INFINITY;
-    for (int cc = 0; cc < n_chunks; ++cc) cm = fmaxf(cm, st_ml[cc * 8 + fj].x);
-    for (int cc = 0; cc < n_chunks; ++cc) {
-      const float2 ml = st_ml[cc * 8 + fj];
-      const float w = part_weight(ml.x, cm);
-      if (w != 0.f) {
-        cl_ += ml.y * w;
-        const float4* src = reinterpret_cast<const float4*>(st_o + (cc * 8 + fj) * D + fd);
+    ptx::mbar_arrive_expect_tx(&bars[0], Q_BYTES);
+    ptx::bulk_load(R0, qsrc, Q_BYTES, &bars[0], ptx::policy_evict_last());
+    issued |= 1u;
+  }
+
+  // Thread tid reads TMEM lane tid: query q = tid / 2, its hi part (pt = 0)
+  // or lo part (pt = 1); it keeps keys [64 pt, 64 pt + 64) of S and dims
+  // [DH pt, DH pt + DH) of O.
+  const int q = tid >> 1, pt = tid & 1;
+  const int qg = qt * kQT + q;
+  const int lim = qg < qn ? L + qg / G : -1;
+  float m = -INFINITY, l = 0.f;
+  float o[DH];  // written by the second product's read-out; pushed only then
+  auto wait_all = [&](bool ok, int bar) {
+    return ptx::group_all(ok && ptx::mbar_wait(&bars[bar], 0, a.timeout_ns), 1, 128);
+  };
+  bool ok = true;
+  if (active) {
+    ok = wait_all(wait_all(true, 0), 1);
+    // S = Q K^T in halves of d: region h of Q and of K, one accumulation chain
 #pragma unroll
-        for (int u = 0; u < DT / 4; ++u) {
-          const float4 v = src[u];
-          co[4 * u + 0] += v.x * w;
-          co[4 * u + 1] += v.y * w;
-          co[4 * u + 2] += v.z * w;
-          co[4 * u + 3] += v.w * w;
+    for (int h = 0; h < NR; ++h) {
+      if (h > 0) {
+        if (ok && tid == 0) load_k(h, 3);  // over the region the first half consumed
+        ok = wait_all(ok, 3);
+      }
+      if (ok && tid == 0) {
+        ptx::tc_fence_after();
+        constexpr uint32_t IDESC1 = ptx::idesc_bf16_f32(128, kTile);
+#pragma unroll
+        for (int k4 = 0; k4 < 4; ++k4) {
+          const int kk = 4 * h + k4;
+          const uint64_t ad = ptx::sdesc_sw128(ptx::smem_u32(R0 + h * kRegion)) + 2 * k4;
+          const uint64_t bd = ptx::sdesc_sw128(ptx::smem_u32(RK)) + 2 * k4;
+          ptx::mma_bf16(tmem, ad, bd, IDESC1, kk > 0 ? 1u : 0u);
+        }
+        ptx::mma_commit(&bars[2 + 2 * h]);
+        issued |= 1u << (2 + 2 * h);
+      }
+      ok = wait_all(ok, 2 + 2 * h);
+    }
+    // Q and K are consumed: V comes over Q (from L2) during the softmax
+    if (ok && tid == 0) {
+      ptx::mbar_arrive_expect_tx(&bars[5], NR * kRegion);
+#pragma unroll
+      for (int h = 0; h < NR; ++h) ptx::tma_load_3d(R0 + h * kRegion, &tmV, &bars[5], 64 * h, p0, z, pol);
+      issued |= 1u << 5;
+    }
+    ptx::tc_fence_after();
+    if (ok) {
+      // S = hi + lo of this thread's keys, 16 keys of each half at a time
+      float sv[64];
+#pragma unroll
+      for (int cc = 0; cc < 4; ++cc) {
+        uint32_t k0[16], k1[16];  // keys 16 cc + j and 64 + 16 cc + j
+        ptx::tmem_ld16(tmem + lane_base + 16 * cc, k0);
+        ptx::tmem_ld16(tmem + lane_base + 64 + 16 * cc, k1);
+        ptx::tmem_ld_wait();
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+          const float v0 = __uint_as_float(k0[j]), v1 = __uint_as_float(k1[j]);
+          const float mine = pt ? v1 : v0, other = pt ? v0 : v1;
+          sv[16 * cc + j] = mine + __shfl_xor_sync(0xFFFFFFFFu, other, 1);
+        }
+      }
+      softmax_tail(sv, pt, p0 + 64 * pt, lim, m, l);
+      // P as bf16 hi (row 2q) and lo (row 2q + 1) parts into TMEM over S, two
+      // keys per column, 16 keys (8 columns of each half of the row) at a
+      // time; each lane completes its row with the partner's half of the keys
+#pragma unroll
+      for (int cc = 0; cc < 4; ++cc) {
+        uint32_t hw[8], lw[8], first[8], second[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const float x0 = sv[16 * cc + 2 * j], x1 = sv[16 * cc + 2 * j + 1];
+          const uint32_t b0 = __float_as_uint(x0), b1 = __float_as_uint(x1);
+          hw[j] = (b0 >> 16) | (b1 & 0xFFFF0000u);
+          const __nv_bfloat162 lv = __floats2bfloat162_rn(x0 - __uint_as_float(b0 & 0xFFFF0000u),
+                                                          x1 - __uint_as_float(b1 & 0xFFFF0000u));
+          lw[j] = *reinterpret_cast<const uint32_t*>(&lv);
+        }
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          // the hi lane takes the partner's hi words (keys 64..127), the lo
+          // lane the partner's lo words (keys 0..63)
+          const uint32_t got = __shfl_xor_sync(0xFFFFFFFFu, pt ? hw[j] : lw[j], 1);
+          first[j] = pt ? got : hw[j];
+          second[j] = pt ? lw[j] : got;
+        }
+        ptx::tmem_st_x8(tmem + lane_base + 8 * cc, first);
+        ptx::tmem_st_x8(tmem + lane_base + 32 + 8 * cc, second);
+      }
+      ptx::tmem_st_wait();
+    }
+    ok = wait_all(ok, 5);
+    // values past the call's last key would reach O through 0 * V
+    if (ok) {
+      const int z0 = kend - p0;
+      if (z0 < kTile) {
+        for (int idx = tid; idx < (kTile - z0) * NR * 8; idx += 128) {
+          const int r = z0 + idx / (NR * 8), rest = idx - (idx / (NR * 8)) * (NR * 8);
+          *reinterpret_cast<uint4*>(R0 + (rest >> 3) * kRegion + r * 128 + (rest & 7) * 16) =
+              make_uint4(0, 0, 0, 0);
         }
       }
     }
-    write_out(co, cl_);
-    return;
-  }
-  // eight chunks' values in flight at a time; the first eight are requested
-  // together with every chunk's maximum, so that up to eight chunks take one
-  // memory round trip
-  float4 v[8][DT / 4];
-  float2 ml[8];
-  auto load8 = [&](int c0) {
+    ptx::fence_proxy_async_smem();
+    // O = P V in 64-dim halves into TMEM columns 64..127 (S's second half,
+    // read out above), each read out before the next is written
 #pragma unroll
-    for (int u8 = 0; u8 < 8; ++u8)
-      if (c0 + u8 < n_chunks) {
-        const size_t pc = item * a.chunks_max + c0 + u8;
-        ml[u8] = __ldcg(a.ws_ml + pc * kQT + fr);
-        const float4* src = reinterpret_cast<const float4*>(a.ws_o + (pc * kQT + fr) * D + fd);
+    for (int h = 0; h < NR; ++h) {
+      ptx::tc_fence_before();
+      __syncthreads();
+      if (ok && tid == 0) {
+        ptx::tc_fence_after();
+        constexpr uint32_t IDESC2 = ptx::idesc_bf16_f32(128, 64, true);
 #pragma unroll
-        for (int u = 0; u < DT / 4; ++u) v[u8][u] = __ldcg(src + u);
+        for (int kk = 0; kk < kTile / 16; ++kk) {
+          const uint64_t bd =
+              ptx::sdesc_sw128_mn(ptx::smem_u32(R0 + h * kRegion) + kk * 2048u, kRegion, 1024u);
+          ptx::mma_bf16_ta(tmem + 64, tmem + 8u * kk, bd, IDESC2, kk > 0 ? 1u : 0u);
+        }
+        ptx::mma_commit(&bars[6 + h]);
+        issued |= 1u << (6 + h);
       }
-  };
-  load8(0);
-  float cm = -INFINITY;
-  for (int cc = 8; cc < n_chunks; ++cc)
-    cm = fmaxf(cm, __ldcg(a.ws_ml + (item * a.chunks_max + cc) * kQT + fr).x);
+      ok = wait_all(ok, 6 + h);
+      ptx::tc_fence_after();
+      if (ok) {
 #pragma unroll
-  for (int u8 = 0; u8 < 8; ++u8)
-    if (u8 < n_chunks) cm = fmaxf(cm, ml[u8].x);
-  for (int c0 = 0; c0 < n_chunks; c0 += 8) {
-    if (c0 > 0) load8(c0);
+        for (int cc = 0; cc < 4; ++cc) {
+          uint32_t v16[16];
+          ptx::tmem_ld16(tmem + lane_base + 64 + 16 * cc, v16);
+          ptx::tmem_ld_wait();
+          const int d0 = 64 * h + 16 * cc, owner = d0 / DH;  // compile-time after unrolling
 #pragma unroll
-    for (int u8 = 0; u8 < 8; ++u8)
-      if (c0 + u8 < n_chunks) {
-        const float w = part_weight(ml[u8].x, cm);
-        if (w != 0.f) {
-          cl_ += ml[u8].y * w;
-#pragma unroll
-          for (int u = 0; u < DT / 4; ++u) {
-            co[4 * u + 0] += v[u8][u].x * w;
-            co[4 * u + 1] += v[u8][u].y * w;
-            co[4 * u + 2] += v[u8][u].z * w;
-            co[4 * u + 3] += v[u8][u].w * w;
+          for (int j = 0; j < 16; ++j) {
+            const float v = __uint_as_float(v16[j]);
+            const float x = __shfl_xor_sync(0xFFFFFFFFu, v, 1);
+            if (pt == owner) o[d0 - owner * DH + j] = v + x;
           }
         }
       }
+    }
+    if (!ok) {
+      if (tid == 0) {
+        atomicOr(a.err, kErrTimeout);
+        // no copy or product may still run when TMEM is freed and the CTA ends
+        for (int i = 0; i < 8; ++i)
+          if (issued & (1u << i)) ptx::mbar_wait(&bars[i], 0, ptx::kDrainNs);
+      }
+      m = -INFINITY;  // nothing of this tile is passed on
+    }
   }
-  write_out(co, cl_);
+  // the V image is consumed: the cluster's partials may come into it
+  ptx::cluster_arrive_relaxed();
+  ptx::griddep_launch_dependents();
+  ptx::tc_fence_before();
+  __syncthreads();
+  if (warp == 0) ptx::tmem_dealloc(tmem, 128);
+
+  // ---- the tile partials, pushed to the CTA that folds their rows ----------
+  ptx::cluster_wait();
+  if (active) {
+    const uint32_t dst_rank = (uint32_t)(q >> 3), row = (uint32_t)(q & 7);
+    if (pt == 0)
+      dsmem_st_f2(ptx::dsmem_map(ptx::smem_u32(s_rml + rank * 8 + row), dst_rank), make_float2(m, l));
+    if (m != -INFINITY) {
+      const uint32_t dst =
+          ptx::dsmem_map(ptx::smem_u32(recv + (rank * 8 + row) * D + pt * DH), dst_rank);
+#pragma unroll
+      for (int u = 0; u < DH / 4; ++u)
+        dsmem_st_f4(dst + 16u * u, make_float4(o[4 * u], o[4 * u + 1], o[4 * u + 2], o[4 * u + 3]));
+    }
+  }
+  ptx::cluster_sync();
+  fold_chunk8<D>(a, recv, s_rml, s_flag, sm, kStage4, rank, c, n_tiles, n_chunks, b, g, qt, qn, G,
+                 r0);
 }
 
 // Clusters of 16 resident at once, two CTAs per SM: 14 in a residency probe
@@ -894,6 +1193,30 @@ cudaError_t launch_attn(const CUtensorMap& tk, const CUtensorMap& tv, const Attn
   return cudaLaunchKernelEx(&cfg, attn_tc_kernel<D, NARROW, PAIR>, tk, tv, a);
 }
 
+template <int D>
+cudaError_t launch_attn4(const CUtensorMap& tk, const CUtensorMap& tv, const AttnArgs& a,
+                         int clusters, cudaStream_t st) {
+  constexpr uint32_t smem = attn4_smem();
+  static const cudaError_t attr = cudaFuncSetAttribute(
+      attn_tc4_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (attr != cudaSuccess) return attr;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(clusters * kCluster, a.nkv);
+  cfg.blockDim = dim3(128);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr2[2];
+  attr2[0].id = cudaLaunchAttributeClusterDimension;
+  attr2[0].val.clusterDim.x = kCluster;
+  attr2[0].val.clusterDim.y = 1;
+  attr2[0].val.clusterDim.z = 1;
+  attr2[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr2[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr2;
+  cfg.numAttrs = 2;
+  return cudaLaunchKernelEx(&cfg, attn_tc4_kernel<D>, tk, tv, a);
+}
+
 }  // namespace
 
 int attn_q_tiles(int rows_per_request, int group) {
@@ -947,6 +1270,7 @@ cudaError_t launch_attention_split(const RowMap& m, const Model& md, KvState& kv
   // Narrow: more than kWideClusters clusters of 8.  Pair: every request has
   // at most two chunks, and the clusters of 16 run at once.
   const bool narrow = clusters8 * c.n_kv_heads > kWideClusters;
+  const bool quad = clusters8 * c.n_kv_heads > kNarrowClusters;
   // Measured: the prefetch of V takes 32 µs off a 7B block at L = 15128 (60
   // clusters of 8) and 12 µs at k = 16 (120), but adds 100 µs to a ragged
   // round of 16 requests (about 440 clusters, some nine waves).
@@ -969,13 +1293,15 @@ cudaError_t launch_attention_split(const RowMap& m, const Model& md, KvState& kv
   if (c.head_dim == 128) {
     e = launch_pdl(qkv_finish_kernel<128>, gf, dim3(64), 0, st, a);
     if (e == cudaSuccess)
-      e = narrow ? launch_attn<128, true, false>(kv.tm_kc, kv.tm_vc, a, clusters, st)
+      e = quad     ? launch_attn4<128>(kv.tm_kc, kv.tm_vc, a, clusters, st)
+          : narrow ? launch_attn<128, true, false>(kv.tm_kc, kv.tm_vc, a, clusters, st)
           : pair ? launch_attn<128, false, true>(kv.tm_kc, kv.tm_vc, a, clusters, st)
                  : launch_attn<128, false, false>(kv.tm_kc, kv.tm_vc, a, clusters, st);
   } else {
     e = launch_pdl(qkv_finish_kernel<64>, gf, dim3(32), 0, st, a);
     if (e == cudaSuccess)
-      e = narrow ? launch_attn<64, true, false>(kv.tm_kc, kv.tm_vc, a, clusters, st)
+      e = quad     ? launch_attn4<64>(kv.tm_kc, kv.tm_vc, a, clusters, st)
+          : narrow ? launch_attn<64, true, false>(kv.tm_kc, kv.tm_vc, a, clusters, st)
           : pair ? launch_attn<64, false, true>(kv.tm_kc, kv.tm_vc, a, clusters, st)
                  : launch_attn<64, false, false>(kv.tm_kc, kv.tm_vc, a, clusters, st);
   }

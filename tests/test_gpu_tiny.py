@@ -217,23 +217,34 @@ def test_batch_of_requests_matches_single(pair):
     st.close()
 
 
-def test_attention_layouts_give_the_same_rows(pair):
-    """The attention runs a call in one of three layouts with the same
-    arithmetic: wide (one wave of clusters of 8), wide with clusters of 16
-    folding two 1024-key chunks in one cluster (every request of at most two
-    chunks), and narrow (several waves; V loaded over K).  A batch of six
-    requests of 2, 4, 1, 3, 4 and 4 chunks takes the narrow layout (36
-    clusters of 8 over the two kv heads); each request alone takes a wide
-    one (the two-chunk request: clusters of 16).  Every request's rows agree
-    bit for bit, and the two-chunk request matches the oracle."""
+LAYOUT_BATCHES = {
+    # 2, 4, 1, 3, 4 and 4 chunks: 36 clusters of 8 over the two kv heads
+    "narrow": ([1500, 3100, 300, 2600, 4000, 3900], (4, 2, 6, 0, 3, 5)),
+    # 36 chunks: 72 clusters of 8, more than the narrow layout keeps resident
+    "quad": ([1500, 3100, 300, 2600, 4000, 3900, 3500, 2000, 1000, 3800, 4050, 2500],
+             (4, 2, 6, 0, 3, 5, 1, 7, 2, 0, 4, 3)),
+}
+
+
+@pytest.mark.parametrize("layout", sorted(LAYOUT_BATCHES))
+def test_attention_layouts_give_the_same_rows(pair, layout):
+    """The attention runs a call in one of four layouts with the same
+    arithmetic: wide (clusters of 8, two CTAs per SM), wide with clusters of
+    16 folding two 1024-key chunks in one cluster (every request of at most
+    two chunks), narrow (V loaded over K, three CTAs per SM) and quad (the
+    first product in halves of d, P in TMEM, four CTAs per SM).  A batch of
+    requests takes the narrow or the quad layout (36 or 72 clusters of 8 over
+    the two kv heads); each request alone takes a wide one (the two-chunk
+    request: clusters of 16).  Every request's rows agree bit for bit, and
+    the two-chunk request matches the oracle."""
     import torch
     from synth import device as D
     cfg = pair.cfg
-    lens = [1500, 3100, 300, 2600, 4000, 3900]
+    lens, ks = LAYOUT_BATCHES[layout]
     cap = 4100
     roots = [int(t) for t in W.root_tokens(cfg, len(lens), 7)]
     rng = np.random.default_rng(13)
-    cands = [[int(t) for t in rng.integers(0, cfg.vocab, k)] for k in (4, 2, 6, 0, 3, 5)]
+    cands = [[int(t) for t in rng.integers(0, cfg.vocab, k)] for k in ks]
     st = pair.state(lens, cap, roots)
     gpu = run_gpu_block(st, cfg, cands)
     st.check()
