@@ -111,7 +111,7 @@ struct AttnArgs {
   int lo_row;
   int32_t* err;
   unsigned long long timeout_ns;
-  int v_prefetch;         // narrow: bring each tile's V into L2 with its K
+  int v_prefetch;         // narrow and quad: bring each tile's V into L2 with its K
   // clusters of request b: [cl_start[b], cl_start[b + 1]); n_ch[b] of them per
   // query tile (chunks covering the host's bound of the request's keys)
   int32_t cl_start[kMaxBatch + 1];
@@ -925,11 +925,11 @@ __global__ void __launch_bounds__(128, 4)
     ptx::tma_load_3d(RK, &tmK, &bars[bar], 64 * h, p0, z, pol);
     issued |= 1u << bar;
   };
-  auto prefetch_rest = [&]() {  // the other K regions and V, into L2
+  auto prefetch_rest = [&]() {  // the other K regions (and V, in launches of a few waves) into L2
 #pragma unroll
     for (int h = 1; h < NR; ++h) ptx::tma_prefetch_3d(&tmK, 64 * h, p0, z);
-#pragma unroll
-    for (int h = 0; h < NR; ++h) ptx::tma_prefetch_3d(&tmV, 64 * h, p0, z);
+    if (a.v_prefetch)
+      for (int h = 0; h < NR; ++h) ptx::tma_prefetch_3d(&tmV, 64 * h, p0, z);
   };
   // a tile of entries older than this call does not depend on the finishing
   // kernel: request it before the wait
