@@ -47,7 +47,9 @@
 // images, two CTAs per SM; NARROW, V loaded over K once the first product is
 // done (from L2, where the launch is small enough to prefetch it) and O
 // accumulated over S in TMEM, three CTAs per SM, for launches of more
-// clusters than the wide layout serves well.
+// clusters than the wide layout serves well; and attn_tc4_kernel, four CTAs
+// per SM in 48 KB, for launches of more clusters than the narrow layout
+// keeps resident.
 // Every fold boundary is a fixed absolute key position (128-key tiles,
 // 1024-key chunks), and a fold with a part a row cannot see (fully masked:
 // m = -inf, l = 0, O = 0) leaves it bitwise unchanged, so a row's result does
