@@ -468,6 +468,23 @@ __device__ __forceinline__ void fold_chunk8(const AttnArgs& a, const float* recv
         for (int u = 0; u < DT / 4; ++u) v[u8][u] = __ldcg(src + u);
       }
   };
+  // more chunks than shared memory holds, but no more than eight plus that:
+  // chunks 8.. come into shared memory by copies issued together with the
+  // first eight's loads, so that all of them take one memory round trip
+  const bool hybrid = n_chunks > 8 && n_chunks - 8 <= stage_max;
+  float* st_o = reinterpret_cast<float*>(sm);                          // [chunk - 8][8 rows][D]
+  float2* st_ml = reinterpret_cast<float2*>(sm + stage_max * 8 * D * 4);  // [chunk - 8][8 rows]
+  if (hybrid) {
+    for (int cc = 8; cc < n_chunks; ++cc) {
+      const size_t pc = item * a.chunks_max + cc;
+      const float* src = a.ws_o + (pc * kQT + fr) * D + fd;
+      float* dst = st_o + ((cc - 8) * 8 + fj) * D + fd;
+#pragma unroll
+      for (int u = 0; u < DT / 4; ++u) ptx::cp_async16(dst + 4 * u, src + 4 * u);
+      if ((tid & 15) == 0 && (fj & 1) == 0)
+        ptx::cp_async16(st_ml + (cc - 8) * 8 + fj, a.ws_ml + pc * kQT + fr);
+    }
+  }
   load8(0);
   float cm = -INFINITY;
   for (int cc = 8; cc < n_chunks; ++cc)
@@ -476,6 +493,27 @@ __device__ __forceinline__ void fold_chunk8(const AttnArgs& a, const float* recv
   for (int u8 = 0; u8 < 8; ++u8)
     if (u8 < n_chunks) cm = fmaxf(cm, ml[u8].x);
   for (int c0 = 0; c0 < n_chunks; c0 += 8) {
+    if (hybrid && c0 == 8) {
+      ptx::cp_async_wait_all();
+      __syncthreads();
+      for (int cc = 8; cc < n_chunks; ++cc) {
+        const float2 mlc = st_ml[(cc - 8) * 8 + fj];
+        const float w = part_weight(mlc.x, cm);
+        if (w != 0.f) {
+          cl_ += mlc.y * w;
+          const float4* src = reinterpret_cast<const float4*>(st_o + ((cc - 8) * 8 + fj) * D + fd);
+#pragma unroll
+          for (int u = 0; u < DT / 4; ++u) {
+            const float4 vv = src[u];
+            co[4 * u + 0] += vv.x * w;
+            co[4 * u + 1] += vv.y * w;
+            co[4 * u + 2] += vv.z * w;
+            co[4 * u + 3] += vv.w * w;
+          }
+        }
+      }
+      break;
+    }
     if (c0 > 0) load8(c0);
 #pragma unroll
     for (int u8 = 0; u8 < 8; ++u8)
